@@ -1,0 +1,491 @@
+"""Benchmark of the grouped ternary (W1.58A16) linear hot path on GB300.
+
+One step = one pass of the whole path over one synthetic batch of the Mamba-2
+1.3B in_proj prefill (W fp32 [8512, 2048], g = 128, X bf16 [16384, 2048],
+dY bf16 [16384, 8512]): tq_quantize (absmean scale + ternary codes + packing),
+tq_linear_fwd (Y = X W^T), and the STE backward dX = dY W^ and dW = dY^T X.
+``value`` is the algorithmic TFLOP/s of the three GEMMs (3 x 2 M N K per step)
+over the device time of the whole step, inputs already in HBM; ``e2e`` is the
+same metric through the C ABI with pinned host buffers, host<->device copies of
+every input and output inside the timed region.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+Under torchrun (N > 1) every rank runs its own replica of the step (weak
+scaling, no collective on the data path); rank 0 prints the JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import hashlib
+import io
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+IN_PROJ = (8512, 2048)
+OUT_PROJ = (2048, 4096)
+M_PREFILL = 16384  # batch 8 x seq 2048
+G = 128
+N_LAYERS = 48
+METRIC = "W1.58A16 linear fwd+bwd TFLOP/s"
+WORKLOAD = ("Mamba-2 1.3B in_proj prefill, one step = tq_quantize W[8512,2048] (g=128) + "
+            "tq_linear_fwd + tq_linear_bwd (dX, dW) at M=16384 (batch 8 x seq 2048)")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+# ------------------------------------------------------------------ helpers
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def kernel_hash(files):
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, "paper_2606_18114_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel, files):
+    """DRAM bytes per launch from a committed ncu capture, if the kernel is unchanged."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(kernel)
+    if not e or e.get("source_sha") != kernel_hash(files):
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        rows = [r for r in csv.reader(io.StringIO(self.out or "")) if len(r) >= 9]
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
+        smax = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if "Active" in r[5 + i]})
+        pw = [float(r[3]) for r in rows if r[3].strip().replace(".", "").isdigit()]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(rows),
+                "power_w_max": max(pw) if pw else None}
+
+
+def dist_setup(n_gpus):
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(0)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------ the step
+class Prefill:
+    """Device-resident inputs/outputs of one projection's prefill step."""
+
+    def __init__(self, tq, n, k, m, g, seed):
+        gen = torch.Generator(device="cuda")
+        gen.manual_seed(seed)
+        self.tq, self.n, self.k, self.m, self.g = tq, n, k, m, g
+        self.w = torch.randn((n, k), generator=gen, device="cuda") * 0.02
+        self.x = torch.randn((m, k), generator=gen, device="cuda").to(torch.bfloat16)
+        self.dy = (torch.randn((m, n), generator=gen, device="cuda") * 1e-2).to(torch.bfloat16)
+        self.codes = torch.empty((n, k // 16), dtype=torch.int32, device="cuda")
+        self.s = torch.empty((n, k // g), dtype=torch.float32, device="cuda")
+        self.z = torch.empty((n, k // g), dtype=torch.int32, device="cuda")
+        self.y = torch.empty((m, n), dtype=torch.float32, device="cuda")
+        self.dx = torch.empty((m, k), dtype=torch.float32, device="cuda")
+        self.dw = torch.empty((n, k), dtype=torch.float32, device="cuda")
+
+    @property
+    def flops(self):
+        return 3 * 2.0 * self.m * self.n * self.k
+
+    def quantize_bytes(self):
+        n, k, g = self.n, self.k, self.g
+        return n * k * 4 + n * k // 4 + 2 * 4 * n * k // g
+
+    def step(self, ev=None):
+        tq = self.tq
+        rec = (lambda i: ev[i].record()) if ev is not None else (lambda i: None)
+        rec(0)
+        tq.quantize(self.w, self.g, out=(self.codes, self.s, self.z))
+        rec(1)
+        tq.linear_fwd(self.x, self.codes, self.s, self.g, y=self.y)
+        rec(2)
+        tq.linear_bwd(self.dy, self.x, self.codes, self.s, self.k, self.g, want_dw=False,
+                      dx=self.dx)
+        rec(3)
+        tq.linear_bwd(self.dy, self.x, self.codes, self.s, self.k, self.g, want_dx=False,
+                      dw=self.dw)
+        rec(4)
+
+
+KERNELS = [  # name, source files, event span
+    ("quantize", ["quantize.cu"], (0, 1)),
+    ("fwd", ["ts_gemm.cu", "ptx.cuh"], (1, 2)),
+    ("dx", ["ts_gemm.cu", "ptx.cuh"], (2, 3)),
+    ("dw", ["dw_gemm.cu", "ptx.cuh"], (3, 4)),
+]
+
+
+def time_prefill(p: Prefill, steps, warmup, world):
+    for _ in range(warmup):
+        p.step()
+    torch.cuda.synchronize()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(steps)]
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for i in range(steps):
+        p.step(evs[i])
+    t1.record()
+    torch.cuda.synchronize()
+    barrier(world)
+    total_ms = t0.elapsed_time(t1)
+    per = {}
+    for name, _, (a, b) in KERNELS:
+        per[name] = sum(e[a].elapsed_time(e[b]) for e in evs) / steps
+    p.tq.device_status()
+    return total_ms, per
+
+
+def time_e2e(p: Prefill, steps, warmup):
+    """Same step through the C ABI from pinned host buffers, copies included."""
+    h_w = p.w.cpu().pin_memory()
+    h_x = p.x.cpu().pin_memory()
+    h_dy = p.dy.cpu().pin_memory()
+    h_y = torch.empty(p.y.shape, dtype=p.y.dtype).pin_memory()
+    h_dx = torch.empty(p.dx.shape, dtype=p.dx.dtype).pin_memory()
+    h_dw = torch.empty(p.dw.shape, dtype=p.dw.dtype).pin_memory()
+
+    def one():
+        p.w.copy_(h_w, non_blocking=True)
+        p.x.copy_(h_x, non_blocking=True)
+        p.dy.copy_(h_dy, non_blocking=True)
+        p.step()
+        h_y.copy_(p.y, non_blocking=True)
+        h_dx.copy_(p.dx, non_blocking=True)
+        h_dw.copy_(p.dw, non_blocking=True)
+
+    for _ in range(warmup):
+        one()
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(steps):
+        one()
+    t1.record()
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1) / steps
+    h2d = sum(t.numel() * t.element_size() for t in (h_w, h_x, h_dy))
+    d2h = sum(t.numel() * t.element_size() for t in (h_y, h_dx, h_dw))
+    return ms, h2d, d2h
+
+
+def decode_sweep(tq, m_list, steps, warmup):
+    """Decode forward over all 48 layers' packed in_proj and out_proj (one batched call)."""
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(1234)
+    mats = []
+    for layer in range(N_LAYERS):
+        for (n, k) in (IN_PROJ, OUT_PROJ):
+            w = torch.randn((n, k), generator=gen, device="cuda") * 0.02
+            codes, s, _ = tq.quantize(w, G)
+            mats.append((n, k, codes, s))
+            del w
+    out = {}
+    for m in m_list:
+        items = []
+        for (n, k, codes, s) in mats:
+            x = torch.randn((m, k), generator=gen, device="cuda").to(torch.bfloat16)
+            items.append(dict(x=x, codes=codes, scales=s, g=G,
+                              y=torch.empty((m, n), device="cuda")))
+        for _ in range(warmup):
+            tq.linear_fwd_batched(items, m)
+        torch.cuda.synchronize()
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record()
+        for _ in range(steps):
+            tq.linear_fwd_batched(items, m)
+        t1.record()
+        torch.cuda.synchronize()
+        ms = t0.elapsed_time(t1) / steps
+        nbytes = sum(it["codes"].numel() * 4 + it["scales"].numel() * 4 + it["x"].numel() * 2 +
+                     it["y"].numel() * 4 for it in items)
+        out[f"M={m}"] = {"us": round(ms * 1e3, 2), "GB/s": round(nbytes / ms / 1e6, 1),
+                         "bytes": nbytes}
+    tq.device_status()
+    return out
+
+
+def quantize_sweep(tq, steps, warmup):
+    """tq_quantize over the 96 projections of 48 blocks (the per-step requantize)."""
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(99)
+    ws = [torch.randn(shape, generator=gen, device="cuda") * 0.02
+          for _ in range(N_LAYERS) for shape in (IN_PROJ, OUT_PROJ)]
+    outs = [(torch.empty((w.shape[0], w.shape[1] // 16), dtype=torch.int32, device="cuda"),
+             torch.empty((w.shape[0], w.shape[1] // G), device="cuda"),
+             torch.empty((w.shape[0], w.shape[1] // G), dtype=torch.int32, device="cuda"))
+            for w in ws]
+
+    def run():
+        for w, o in zip(ws, outs):
+            tq.quantize(w, G, out=o)
+
+    for _ in range(warmup):
+        run()
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(steps):
+        run()
+    t1.record()
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1) / steps
+    nbytes = sum(w.numel() * 4 + w.numel() // 4 + 2 * 4 * w.numel() // G for w in ws)
+    tq.device_status()
+    del ws, outs
+    return {"ms": round(ms, 3), "GB/s": round(nbytes / ms / 1e6, 1), "bytes": nbytes}
+
+
+# ------------------------------------------------------------------ oracle (CPU)
+def blas_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return len(os.sched_getaffinity(0))
+
+
+def oracle_sample(seed=0):
+    """A bounded sample of one step, run by the oracle on the host cores.
+
+    Quantises the full W [8512, 2048] and computes Y and dX for 64 token rows and
+    dW for 64 output rows (fp64). Returns (flops of the sample, seconds).
+    """
+    from oracle import tq_oracle as O
+    from paper_2606_18114_gb300 import synth
+    n, k = IN_PROJ
+    w = synth.latent_weights(n, k, seed=seed)
+    rs = np.random.default_rng(seed)
+    rows = 64
+    x = synth.activations_bf16(M_PREFILL, k, seed=seed, stream="x")
+    dy_rows = synth.activations_bf16(rows, n, seed=seed, std=1e-2, stream="dy_sample")
+    nsel = np.sort(rs.choice(n, rows, replace=False))
+    dy_cols = synth.activations_bf16(M_PREFILL, rows, seed=seed, std=1e-2, stream="dy_cols")
+    t0 = time.perf_counter()
+    codes, s, z, _ = O.quantize(w, G)
+    w_hat = O.dequantize(codes, s, k, G)
+    O.linear_fwd(x[:rows], w_hat)
+    O.linear_bwd_dx(dy_rows, w_hat)
+    O.linear_bwd_dw(dy_cols, x)
+    dt = time.perf_counter() - t0
+    flops = 2.0 * rows * n * k * 2 + 2.0 * rows * M_PREFILL * k
+    del nsel
+    return flops, dt
+
+
+def cpu_baseline():
+    flops, dt = oracle_sample()
+    return {"value": round(flops / dt / 1e12, 6), "unit": "TFLOP/s", "cores": blas_threads(),
+            "kind": "oracle",
+            "sample": ("oracle (numpy, fp64) on one step's bounded sample: quantize the full "
+                       "W[8512,2048] g=128, then Y and dX for 64 of 16384 token rows and dW for "
+                       "64 of 8512 output rows; flops of the sample / wall time"),
+            "seconds": round(dt, 2)}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    for _ in range(args.warmup):
+        oracle_sample()
+    times, flops = [], 0.0
+    for _ in range(args.steps):
+        f, dt = oracle_sample()
+        flops, times = f, times + [dt]
+    dt = sum(times) / len(times)
+    value = flops / dt / 1e12
+    line = {
+        "metric": METRIC, "value": round(value, 6), "unit": "TFLOP/s", "impl": "reference",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(dt * 1e3, 1), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "M": M_PREFILL, "N": IN_PROJ[0], "K": IN_PROJ[1],
+                   "g": G, "sample": "bounded oracle sample per step (see cpu_baseline)"},
+        "cpu_baseline": {"value": round(value, 6), "unit": "TFLOP/s", "cores": blas_threads(),
+                         "kind": "oracle",
+                         "sample": "quantize full W; Y, dX on 64 token rows; dW on 64 output rows"},
+        "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------ main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="tq", choices=["tq", "reference"])
+    ap.add_argument("--no-extra", action="store_true", help="skip decode/quantize sweeps")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+    if args.warmup < 3:
+        args.warmup = 3
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_18114_gb300 import tq
+
+    rank, world, local = dist_setup(args.gpus)
+    p = Prefill(tq, IN_PROJ[0], IN_PROJ[1], M_PREFILL, G, seed=1000 + rank)
+    with ClockSampler(local) as clk:
+        total_ms, per = time_prefill(p, args.steps, args.warmup, world)
+    total_ms = max_over_ranks(total_ms, world)
+    ms = total_ms / args.steps
+    value = world * p.flops / (ms * 1e-3) / 1e12
+
+    pk, pk_kind = peaks()
+    gemm_flops = 2.0 * p.m * p.n * p.k
+    kinfo = {}
+    for name, files, _ in KERNELS:
+        t = per[name]
+        if name == "quantize":
+            ach = p.quantize_bytes() / (t * 1e-3) / 1e9
+            kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "GB/s",
+                           "frac": round(ach / pk["hbm_gbs"], 4)}
+        else:
+            ach = gemm_flops / (t * 1e-3) / 1e12
+            kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "TFLOP/s",
+                           "frac": round(ach / pk["bf16_tflops"], 4)}
+    dom = max((n for n, _, _ in KERNELS if n != "quantize"), key=lambda n: per[n])
+    dom_files = dict((n, f) for n, f, _ in KERNELS)[dom]
+    roof = {"kernel": dom, "bound": "tensor", "achieved": kinfo[dom]["achieved"],
+            "peak": pk["bf16_tflops"], "unit": "TFLOP/s", "frac": kinfo[dom]["frac"],
+            "traffic": recorded_traffic(dom, dom_files),
+            "peak_kind": f"{pk_kind} bf16 dense (burst)",
+            "algorithmic_per_launch": gemm_flops}
+
+    e2e_ms, h2d, d2h = time_e2e(p, max(5, args.steps // 10), 2)
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD, "M": M_PREFILL, "N": IN_PROJ[0], "K": IN_PROJ[1],
+                   "g": G, "w_dist": "N(0,0.02^2)", "x_dist": "N(0,1) bf16",
+                   "dy_dist": "N(0,1e-2^2) bf16", "outputs": "Y, dX fp32; dW fp32",
+                   "l2": "no flush: every step reads and writes > 1 GB (inputs exceed the 129 MB L2)",
+                   "replicas": world},
+        "roofline": roof,
+        "kernels": kinfo,
+        "e2e": {"value": round(world * p.flops / (e2e_ms * 1e-3) / 1e12, 2), "unit": "TFLOP/s",
+                "ms_per_step": round(e2e_ms, 3), "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": 4 * args.steps,
+        "clocks": clk.summary(),
+    }
+    if not args.no_extra and rank == 0:
+        line["extra"] = {
+            "decode_48_layers": decode_sweep(tq, (1, 4, 16), 20, 3),
+            "quantize_48_layers_g128": quantize_sweep(tq, 5, 2),
+            "hbm_peak_gbs": pk["hbm_gbs"],
+        }
+    if rank == 0 and world == 1 and not args.no_cpu:
+        line["cpu_baseline"] = cpu_baseline()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,158 @@
+/*
+ * tq.h — C ABI of the grouped ternary (W1.58A16) linear layer on GB300 (sm_103a).
+ *
+ * The layer is the TernaryLinear of "Ternary Mamba: Grouped Quantization-Aware
+ * Training of W1.58A16 State Space Models", §3.1: latent fp32 weights W [N, K]
+ * (N = out_features, K = in_features) are split into groups of g consecutive
+ * elements along K inside one row; each group gets the non-learned scale
+ * s = mean |w| (recomputed at every call), codes round(clip(w / s, -1, 1)) in
+ * {-1, 0, +1}, and the dequantised weight s * code. The forward product uses
+ * 16-bit (bf16) activations; the backward is the straight-through estimator.
+ *
+ * Conventions for every entry point
+ *   - Every pointer is DEVICE memory owned by the caller, contiguous row-major,
+ *     16-byte aligned. The library keeps no pointer after a call returns.
+ *   - Work is enqueued on `stream` (a cudaStream_t passed as void*; NULL is the
+ *     legacy default stream). No entry point synchronises, except
+ *     tq_device_status(). No entry point allocates device memory.
+ *   - Arguments are checked before anything is enqueued. A rejected call
+ *     returns TQ_ERR_INVALID_ARG or TQ_ERR_UNSUPPORTED, writes nothing and
+ *     leaves a message in tq_last_error().
+ *   - A failed launch returns TQ_ERR_CUDA. Kernels bound every wait they
+ *     make; a wait that runs out records TQ_ERR_TIMEOUT in a per-device status
+ *     word that tq_device_status() returns (and clears). Outputs of such a
+ *     call are undefined.
+ *   - Sizes of zero are allowed and do nothing (except that dW is zeroed by
+ *     tq_linear_bwd when M = 0 and accumulate_dw = 0).
+ *   - Group sizes: g in {32, 64, 128, 256, 512}.
+ *
+ * Packed code layout (2 bits per weight; the paper asks only for "packed
+ * 2-bit weight storage", §8 — this particular layout is this library's)
+ *   codes is uint32 [N][K/16]; word w of row n holds k in [16w, 16w + 16).
+ *   Code i = k % 16 sits at bit 2*(i/2) when i is even and at bit
+ *   16 + 2*(i/2) when i is odd (even codes fill the low half-word, odd codes
+ *   the high half-word, pair j = (2j, 2j+1) at bits 2j and 16+2j).
+ *   Values: 0b00 -> 0, 0b01 -> +1, 0b11 -> -1; 0b10 is never written.
+ *   With this layout a shift and a mask turn one pair into a bf16x2 holding
+ *   (2*c_2j, 2*c_2j+1), because the 2-bit value v times 0x4000 is the bf16 bit
+ *   pattern of 0, +2.0 or -2.0.
+ *
+ * Scales are fp32 [N][K/g]; zero counts are int32 [N][K/g].
+ */
+#ifndef TQ_H_
+#define TQ_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define TQ_API __attribute__((visibility("default")))
+#else
+#define TQ_API
+#endif
+
+typedef enum {
+  TQ_OK = 0,
+  TQ_ERR_INVALID_ARG = 1, /* null/misaligned pointer, bad size or group size   */
+  TQ_ERR_UNSUPPORTED = 2, /* valid request outside what the kernels handle      */
+  TQ_ERR_CUDA = 3,        /* CUDA runtime or launch error                       */
+  TQ_ERR_TIMEOUT = 4      /* a device-side wait ran out (tq_device_status only) */
+} tq_status;
+
+typedef enum {
+  TQ_OUT_F32 = 0,  /* fp32 output (default: keeps the max-element error small) */
+  TQ_OUT_BF16 = 1  /* bf16 output, round to nearest even                        */
+} tq_out_dtype;
+
+/*
+ * tq_quantize — §3.1 quantiser: per-group absmean scale, ternary codes, packing.
+ *   w            fp32 [n][k], latent weights (read only).
+ *   n, k         n >= 0; k >= 0, k % 16 == 0 and k % g == 0.
+ *   g            group size along k.
+ *   codes        out: uint32 [n][k/16], layout above.
+ *   scales       out: fp32 [n][k/g], s = (1/g) * sum |w| over the group.
+ *   zero_counts  out: int32 [n][k/g], number of zero codes in the group
+ *                (the zero-ratio monitor of §4).
+ * The code of w is +-1 when |w / s| > 0.5 with the division in fp32 (round
+ * half to even sends 0.5 to 0), 0 otherwise; a group with s = 0 is all zeros.
+ * Inputs must be finite.
+ */
+TQ_API tq_status tq_quantize(const float* w, int64_t n, int64_t k, int32_t g,
+                      uint32_t* codes, float* scales, int32_t* zero_counts,
+                      void* stream);
+
+/*
+ * tq_linear_fwd — W1.58A16 forward (§3.1, "W1.58A16" of the title):
+ *   y[m][n] = sum_k x[m][k] * s[n][k/g] * code[n][k].
+ *   x            bf16 [m][k] activations.
+ *   codes/scales as produced by tq_quantize for W [n][k].
+ *   y            out: [m][n], fp32 (TQ_OUT_F32) or bf16 (TQ_OUT_BF16).
+ *   Requires k % 64 == 0 and k % g == 0; n >= 1 when m >= 1.
+ *   m <= 16 runs the decode kernel, larger m the tensor-core GEMM; both expand
+ *   the codes on chip to bf16 (bf16(s) * code) and accumulate in fp32.
+ */
+TQ_API tq_status tq_linear_fwd(const void* x, int64_t m, int64_t k,
+                        const uint32_t* codes, const float* scales, int64_t n, int32_t g,
+                        void* y, int32_t y_dtype, void* stream);
+
+/*
+ * tq_linear_bwd — straight-through-estimator backward (§3.1; STE = identity
+ * through round and clip, no gradient to the non-learned scale):
+ *   dx[m][k] = sum_n dy[m][n] * s[n][k/g] * code[n][k]      (through W^)
+ *   dw[n][k] = sum_m dy[m][n] * x[m][k]                     (to latent W)
+ *   dy           bf16 [m][n]; x bf16 [m][k] (the forward's input).
+ *   dx           out: [m][k], fp32 or bf16 (dx_dtype); NULL skips dX.
+ *   dw           out: fp32 [n][k]; NULL skips dW. accumulate_dw != 0 adds to
+ *                dw instead of overwriting it.
+ *   Requires k % 64 == 0, k % g == 0, n % 8 == 0. x may be NULL when dw is.
+ */
+TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t n, int64_t k,
+                        const uint32_t* codes, const float* scales, int32_t g,
+                        void* dx, int32_t dx_dtype, float* dw, int32_t accumulate_dw,
+                        void* stream);
+
+/* One matrix of a batched decode call (tq_linear_fwd_batched). */
+typedef struct {
+  const void* x;          /* bf16 [m][k]                         */
+  const uint32_t* codes;  /* uint32 [n][k/16]                    */
+  const float* scales;    /* fp32 [n][k/g]                       */
+  void* y;                /* [m][n], dtype y_dtype               */
+  int64_t n;              /* out_features                        */
+  int64_t k;              /* in_features, k % 64 == 0            */
+  int32_t g;              /* group size                          */
+  int32_t y_dtype;        /* tq_out_dtype                        */
+} tq_fwd_desc;
+
+#define TQ_MAX_BATCH 256
+
+/*
+ * tq_linear_fwd_batched — the decode forward of many matrices in one launch
+ * (e.g. every in_proj and out_proj of a 48-block model for one token step):
+ * for each i < count, y_i = x_i W^_i^T exactly as tq_linear_fwd, all with the
+ * same token count m (1 <= m <= 16). descs is a HOST array (copied into the
+ * launch; not kept); count <= TQ_MAX_BATCH.
+ */
+TQ_API tq_status tq_linear_fwd_batched(const tq_fwd_desc* descs, int32_t count, int64_t m,
+                                void* stream);
+
+/*
+ * tq_device_status — synchronises `stream`, then returns and clears the status
+ * word of the current device: TQ_OK, or TQ_ERR_TIMEOUT if a kernel's bounded
+ * wait ran out since the last call; TQ_ERR_CUDA if the synchronise failed.
+ */
+TQ_API tq_status tq_device_status(void* stream);
+
+/* Message of the last failure on the calling thread ("" if none). */
+TQ_API const char* tq_last_error(void);
+
+/* Library version string. */
+TQ_API const char* tq_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TQ_H_ */

@@ -1,0 +1,59 @@
+// kernels.cuh — launchers of the sm_103a kernels (internal to libtq).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace tq {
+
+// quantize.cu ----------------------------------------------------------------
+cudaError_t launch_quantize(const float* w, int64_t n, int64_t k, int g, uint32_t* codes,
+                            float* scales, int32_t* zeros, int num_sms, cudaStream_t stream);
+
+// ts_gemm.cu -----------------------------------------------------------------
+// Ternary x bf16 products with the expanded ternary weights as the tensor-memory
+// A operand. kTsFwd: out[m][n] = sum_k x[m][k] w^[n][k] (B = x, rows = n).
+// kTsDx: out[m][k] = sum_n dy[m][n] w^[n][k] (B = dy, rows = k).
+enum TsMode : int { kTsFwd = 0, kTsDx = 1 };
+
+struct TsArgs {
+  const uint32_t* codes;  // uint32 [wn][wk/16]
+  const float* scales;    // fp32 [wn][wk/g]
+  void* out;              // [m][rows], fp32 or bf16
+  int* status;            // device status word (timeouts)
+  int64_t wn, wk;         // shape of the latent weight matrix W [wn][wk]
+  int64_t m;              // tokens
+  int32_t log2g;          // log2 of the group size
+  int32_t out_bf16;       // 1: bf16 output
+};
+
+// Tile of the activation operand along the token dimension.
+int ts_tile_tokens(int64_t m);
+size_t ts_smem_bytes(int bn);
+
+// tmap_b: bf16 activations [m][red] with box {64, bn}, 128-byte swizzle.
+// tmap_codes: uint32 codes [wn][wk/16] with box {4, 128} (fwd) or {8, 64} (dx).
+cudaError_t launch_ts_gemm(int mode, int bn, const CUtensorMap& tmap_b,
+                           const CUtensorMap& tmap_codes, const TsArgs& args,
+                           cudaStream_t stream);
+
+// dw_gemm.cu -----------------------------------------------------------------
+// dW[n][k] (+)= sum_m dy[m][n] x[m][k], both operands MN-major from TMA.
+struct DwArgs {
+  float* dw;       // fp32 [n][k]
+  int* status;
+  int64_t m, n, k;
+  int32_t accumulate;
+};
+
+constexpr int kDwTileK = 128;  // lanes: input features
+constexpr int kDwTileN = 256;  // columns: output features
+size_t dw_smem_bytes();
+
+// tmap_x: bf16 x [m][k] box {64, 64}; tmap_dy: bf16 dy [m][n] box {64, 64};
+// both with the 128-byte swizzle.
+cudaError_t launch_dw_gemm(const CUtensorMap& tmap_x, const CUtensorMap& tmap_dy,
+                           const DwArgs& args, cudaStream_t stream);
+
+}  // namespace tq

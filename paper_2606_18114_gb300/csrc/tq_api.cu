@@ -1,0 +1,370 @@
+// tq_api.cu — the C ABI of include/tq.h: argument checks, TMA descriptors, dispatch.
+//
+// Nothing here computes the method: every step runs in the kernels of
+// quantize.cu, ts_gemm.cu and dw_gemm.cu. This file only validates arguments,
+// encodes tensor maps for the operands, and enqueues launches on the caller's
+// stream.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdarg.h>
+#include <stdint.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "kernels.cuh"
+#include "tq.h"
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+tq_status fail(tq_status st, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return st;
+}
+
+tq_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(TQ_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// Status word written by kernels whose bounded waits run out (one per device).
+__device__ int g_device_status;
+
+struct DeviceInfo {
+  bool ready = false;
+  int num_sms = 0;
+  int* status = nullptr;
+};
+
+constexpr int kMaxDevices = 64;
+DeviceInfo g_devices[kMaxDevices];
+std::mutex g_devices_mu;
+
+tq_status device_info(const DeviceInfo** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return fail(TQ_ERR_UNSUPPORTED, "device %d", dev);
+  std::lock_guard<std::mutex> lock(g_devices_mu);
+  DeviceInfo& d = g_devices[dev];
+  if (!d.ready) {
+    int major = 0, minor = 0, sms = 0;
+    if ((e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+      return cuda_fail(e, "cudaDeviceGetAttribute");
+    if (major != 10 || minor != 3)
+      return fail(TQ_ERR_UNSUPPORTED, "libtq is built for sm_103a (GB300); device %d is sm_%d%d",
+                  dev, major, minor);
+    void* p = nullptr;
+    if ((e = cudaGetSymbolAddress(&p, g_device_status)) != cudaSuccess)
+      return cuda_fail(e, "cudaGetSymbolAddress");
+    d.num_sms = sms;
+    d.status = static_cast<int*>(p);
+    d.ready = true;
+  }
+  *out = &d;
+  return TQ_OK;
+}
+
+// ---------------------------------------------------------------- tensor maps
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// 2-D row-major tensor [outer][inner] with a box of [box_outer][box_inner].
+tq_status make_map(CUtensorMap* map, CUtensorMapDataType dt, int elem_bytes, const void* base,
+                   int64_t inner, int64_t outer, uint32_t box_inner, uint32_t box_outer,
+                   CUtensorMapSwizzle swz) {
+  EncodeTiledFn fn = encode_fn();
+  if (fn == nullptr) return fail(TQ_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(outer)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(inner) * elem_bytes};
+  const cuuint32_t box[2] = {box_inner, box_outer};
+  const cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(TQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+  return TQ_OK;
+}
+
+// ---------------------------------------------------------------- checks
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int log2_group(int32_t g) {
+  switch (g) {
+    case 32: return 5;
+    case 64: return 6;
+    case 128: return 7;
+    case 256: return 8;
+    case 512: return 9;
+    default: return -1;
+  }
+}
+
+constexpr int64_t kMaxDim = (int64_t(1) << 31) - 1;  // TMA coordinates are int32
+
+tq_status check_ptr(const void* p, const char* name) {
+  if (p == nullptr) return fail(TQ_ERR_INVALID_ARG, "%s is NULL", name);
+  if (!aligned16(p)) return fail(TQ_ERR_INVALID_ARG, "%s is not 16-byte aligned", name);
+  return TQ_OK;
+}
+
+#define TQ_TRY(expr)                 \
+  do {                               \
+    const tq_status st_ = (expr);    \
+    if (st_ != TQ_OK) return st_;    \
+  } while (0)
+
+tq_status check_linear_shape(int64_t m, int64_t n, int64_t k, int32_t g) {
+  if (m < 0 || n < 0 || k < 0)
+    return fail(TQ_ERR_INVALID_ARG, "negative size (m=%lld n=%lld k=%lld)", (long long)m,
+                (long long)n, (long long)k);
+  if (log2_group(g) < 0) return fail(TQ_ERR_INVALID_ARG, "group size %d not in {32..512}", g);
+  if (k % g != 0) return fail(TQ_ERR_INVALID_ARG, "k=%lld is not a multiple of g=%d", (long long)k, g);
+  if (k % 64 != 0)
+    return fail(TQ_ERR_UNSUPPORTED, "k=%lld: the linear kernels need k %% 64 == 0", (long long)k);
+  if (m > kMaxDim || n > kMaxDim || k > kMaxDim)
+    return fail(TQ_ERR_UNSUPPORTED, "dimension above 2^31-1");
+  return TQ_OK;
+}
+
+tq_status fwd_checked(const void* x, int64_t m, int64_t k, const uint32_t* codes,
+                      const float* scales, int64_t n, int32_t g, void* y, int32_t y_dtype,
+                      cudaStream_t stream, const tq::TsArgs* proto) {
+  if (m == 0 || n == 0) return TQ_OK;
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  const size_t ybytes = y_dtype == TQ_OUT_BF16 ? 2 : 4;
+  if (k == 0) {
+    cudaError_t e = cudaMemsetAsync(y, 0, static_cast<size_t>(m) * n * ybytes, stream);
+    return e == cudaSuccess ? TQ_OK : cuda_fail(e, "cudaMemsetAsync");
+  }
+  const int bn = tq::ts_tile_tokens(m);
+  if ((m + bn - 1) / bn > 65535) return fail(TQ_ERR_UNSUPPORTED, "m=%lld too large", (long long)m);
+  if ((n + 127) / 128 > 2147483647LL) return fail(TQ_ERR_UNSUPPORTED, "n too large");
+  CUtensorMap tb, tc;
+  TQ_TRY(make_map(&tb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, x, k, m, 64, bn,
+                  CU_TENSOR_MAP_SWIZZLE_128B));
+  TQ_TRY(make_map(&tc, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, codes, k / 16, n, 4, 128,
+                  CU_TENSOR_MAP_SWIZZLE_NONE));
+  tq::TsArgs a = *proto;
+  a.codes = codes;
+  a.scales = scales;
+  a.out = y;
+  a.status = dev->status;
+  a.wn = n;
+  a.wk = k;
+  a.m = m;
+  a.log2g = log2_group(g);
+  a.out_bf16 = y_dtype == TQ_OUT_BF16;
+  cudaError_t e = tq::launch_ts_gemm(tq::kTsFwd, bn, tb, tc, a, stream);
+  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "forward launch");
+}
+
+tq_status check_fwd_args(const void* x, int64_t m, int64_t k, const uint32_t* codes,
+                         const float* scales, int64_t n, int32_t g, const void* y,
+                         int32_t y_dtype) {
+  TQ_TRY(check_linear_shape(m, n, k, g));
+  if (y_dtype != TQ_OUT_F32 && y_dtype != TQ_OUT_BF16)
+    return fail(TQ_ERR_INVALID_ARG, "y_dtype %d", y_dtype);
+  if (m == 0 || n == 0) return TQ_OK;
+  TQ_TRY(check_ptr(y, "y"));
+  if (k == 0) return TQ_OK;
+  TQ_TRY(check_ptr(x, "x"));
+  TQ_TRY(check_ptr(codes, "codes"));
+  TQ_TRY(check_ptr(scales, "scales"));
+  return TQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+TQ_API const char* tq_last_error(void) { return g_err; }
+
+TQ_API const char* tq_version(void) { return "tq 0.1 (sm_103a)"; }
+
+TQ_API tq_status tq_quantize(const float* w, int64_t n, int64_t k, int32_t g, uint32_t* codes,
+                             float* scales, int32_t* zero_counts, void* stream) {
+  g_err[0] = 0;
+  if (n < 0 || k < 0) return fail(TQ_ERR_INVALID_ARG, "negative size");
+  if (log2_group(g) < 0) return fail(TQ_ERR_INVALID_ARG, "group size %d not in {32..512}", g);
+  if (k % 16 != 0) return fail(TQ_ERR_INVALID_ARG, "k=%lld is not a multiple of 16", (long long)k);
+  if (k % g != 0) return fail(TQ_ERR_INVALID_ARG, "k=%lld is not a multiple of g=%d", (long long)k, g);
+  if (n == 0 || k == 0) return TQ_OK;
+  if (n > INT64_MAX / k) return fail(TQ_ERR_INVALID_ARG, "n*k overflows");
+  TQ_TRY(check_ptr(w, "w"));
+  TQ_TRY(check_ptr(codes, "codes"));
+  TQ_TRY(check_ptr(scales, "scales"));
+  TQ_TRY(check_ptr(zero_counts, "zero_counts"));
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaError_t e = tq::launch_quantize(w, n, k, g, codes, scales, zero_counts, dev->num_sms,
+                                      static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "quantize launch");
+}
+
+TQ_API tq_status tq_linear_fwd(const void* x, int64_t m, int64_t k, const uint32_t* codes,
+                               const float* scales, int64_t n, int32_t g, void* y,
+                               int32_t y_dtype, void* stream) {
+  g_err[0] = 0;
+  TQ_TRY(check_fwd_args(x, m, k, codes, scales, n, g, y, y_dtype));
+  tq::TsArgs proto{};
+  return fwd_checked(x, m, k, codes, scales, n, g, y, y_dtype, static_cast<cudaStream_t>(stream),
+                     &proto);
+}
+
+TQ_API tq_status tq_linear_fwd_batched(const tq_fwd_desc* descs, int32_t count, int64_t m,
+                                       void* stream) {
+  g_err[0] = 0;
+  if (count < 0 || count > TQ_MAX_BATCH)
+    return fail(TQ_ERR_INVALID_ARG, "count %d not in [0, %d]", count, TQ_MAX_BATCH);
+  if (count == 0) return TQ_OK;
+  if (descs == nullptr) return fail(TQ_ERR_INVALID_ARG, "descs is NULL");
+  if (m < 1 || m > 16) return fail(TQ_ERR_INVALID_ARG, "batched decode needs 1 <= m <= 16");
+  for (int32_t i = 0; i < count; ++i) {
+    const tq_fwd_desc& d = descs[i];
+    const tq_status st = check_fwd_args(d.x, m, d.k, d.codes, d.scales, d.n, d.g, d.y, d.y_dtype);
+    if (st != TQ_OK) {
+      char msg[512];
+      snprintf(msg, sizeof(msg), "descs[%d]: %s", i, g_err);
+      return fail(st, "%s", msg);
+    }
+  }
+  tq::TsArgs proto{};
+  for (int32_t i = 0; i < count; ++i) {
+    const tq_fwd_desc& d = descs[i];
+    TQ_TRY(fwd_checked(d.x, m, d.k, d.codes, d.scales, d.n, d.g, d.y, d.y_dtype,
+                       static_cast<cudaStream_t>(stream), &proto));
+  }
+  return TQ_OK;
+}
+
+TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t n, int64_t k,
+                               const uint32_t* codes, const float* scales, int32_t g, void* dx,
+                               int32_t dx_dtype, float* dw, int32_t accumulate_dw, void* stream) {
+  g_err[0] = 0;
+  TQ_TRY(check_linear_shape(m, n, k, g));
+  if (n % 8 != 0)
+    return fail(TQ_ERR_UNSUPPORTED, "n=%lld: the backward kernels need n %% 8 == 0", (long long)n);
+  if (dx_dtype != TQ_OUT_F32 && dx_dtype != TQ_OUT_BF16)
+    return fail(TQ_ERR_INVALID_ARG, "dx_dtype %d", dx_dtype);
+  if (dx == nullptr && dw == nullptr) return fail(TQ_ERR_INVALID_ARG, "dx and dw are both NULL");
+  const bool want_dx = dx != nullptr && m > 0 && k > 0;
+  const bool want_dw = dw != nullptr && n > 0 && k > 0;
+  if (want_dx) {
+    TQ_TRY(check_ptr(dx, "dx"));
+    if (n > 0) {
+      TQ_TRY(check_ptr(dy, "dy"));
+      TQ_TRY(check_ptr(codes, "codes"));
+      TQ_TRY(check_ptr(scales, "scales"));
+    }
+  }
+  if (want_dw) {
+    TQ_TRY(check_ptr(dw, "dw"));
+    if (m > 0) {
+      TQ_TRY(check_ptr(dy, "dy"));
+      TQ_TRY(check_ptr(x, "x"));
+    }
+  }
+  if (!want_dx && !want_dw) return TQ_OK;
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+
+  if (want_dx) {
+    const size_t dxb = dx_dtype == TQ_OUT_BF16 ? 2 : 4;
+    if (n == 0) {
+      cudaError_t e = cudaMemsetAsync(dx, 0, static_cast<size_t>(m) * k * dxb, st);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+    } else {
+      const int bn = tq::ts_tile_tokens(m);
+      if ((m + bn - 1) / bn > 65535) return fail(TQ_ERR_UNSUPPORTED, "m too large");
+      CUtensorMap tb, tc;
+      TQ_TRY(make_map(&tb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, dy, n, m, 64, bn,
+                      CU_TENSOR_MAP_SWIZZLE_128B));
+      TQ_TRY(make_map(&tc, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, codes, k / 16, n, 8, 64,
+                      CU_TENSOR_MAP_SWIZZLE_NONE));
+      tq::TsArgs a{};
+      a.codes = codes;
+      a.scales = scales;
+      a.out = dx;
+      a.status = dev->status;
+      a.wn = n;
+      a.wk = k;
+      a.m = m;
+      a.log2g = log2_group(g);
+      a.out_bf16 = dx_dtype == TQ_OUT_BF16;
+      cudaError_t e = tq::launch_ts_gemm(tq::kTsDx, bn, tb, tc, a, st);
+      if (e != cudaSuccess) return cuda_fail(e, "dX launch");
+    }
+  }
+  if (want_dw) {
+    if (m == 0) {
+      if (!accumulate_dw) {
+        cudaError_t e = cudaMemsetAsync(dw, 0, static_cast<size_t>(n) * k * 4, st);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+      }
+    } else {
+      if ((n + tq::kDwTileN - 1) / tq::kDwTileN > 65535)
+        return fail(TQ_ERR_UNSUPPORTED, "n too large");
+      CUtensorMap tx, tdy;
+      TQ_TRY(make_map(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, x, k, m, 64, 64,
+                      CU_TENSOR_MAP_SWIZZLE_128B));
+      TQ_TRY(make_map(&tdy, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, dy, n, m, 64, 64,
+                      CU_TENSOR_MAP_SWIZZLE_128B));
+      tq::DwArgs a{};
+      a.dw = dw;
+      a.status = dev->status;
+      a.m = m;
+      a.n = n;
+      a.k = k;
+      a.accumulate = accumulate_dw != 0;
+      cudaError_t e = tq::launch_dw_gemm(tx, tdy, a, st);
+      if (e != cudaSuccess) return cuda_fail(e, "dW launch");
+    }
+  }
+  return TQ_OK;
+}
+
+TQ_API tq_status tq_device_status(void* stream) {
+  g_err[0] = 0;
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  int v = 0;
+  if ((e = cudaMemcpy(&v, dev->status, sizeof(int), cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "status read");
+  if (v != 0) {
+    const int zero = 0;
+    if ((e = cudaMemcpy(dev->status, &zero, sizeof(int), cudaMemcpyHostToDevice)) != cudaSuccess)
+      return cuda_fail(e, "status clear");
+    return fail(TQ_ERR_TIMEOUT, "a kernel wait ran out (device status %d)", v);
+  }
+  return TQ_OK;
+}
+
+}  // extern "C"

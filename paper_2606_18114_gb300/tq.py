@@ -1,0 +1,184 @@
+"""ctypes binding of libtq (include/tq.h), with the same entry-point names.
+
+Argument marshalling only: torch supplies device memory and the current CUDA
+stream, every step of the computation runs in libtq's sm_103a kernels. There is
+no fallback: if libtq.so is missing or fails to load, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import torch
+
+__all__ = [
+    "TqError",
+    "load",
+    "quantize",
+    "linear_fwd",
+    "linear_bwd",
+    "linear_fwd_batched",
+    "device_status",
+    "version",
+    "OUT_F32",
+    "OUT_BF16",
+    "EXPORTS",
+]
+
+OUT_F32 = 0
+OUT_BF16 = 1
+STATUS = {0: "TQ_OK", 1: "TQ_ERR_INVALID_ARG", 2: "TQ_ERR_UNSUPPORTED", 3: "TQ_ERR_CUDA",
+          4: "TQ_ERR_TIMEOUT"}
+# Every symbol include/tq.h declares.
+EXPORTS = ("tq_quantize", "tq_linear_fwd", "tq_linear_bwd", "tq_linear_fwd_batched",
+           "tq_device_status", "tq_last_error", "tq_version")
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtq.so")
+_lib = None
+
+
+class TqError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS.get(status, status)}: {message}")
+        self.status = status
+
+
+class FwdDesc(ctypes.Structure):
+    _fields_ = [
+        ("x", ctypes.c_void_p),
+        ("codes", ctypes.c_void_p),
+        ("scales", ctypes.c_void_p),
+        ("y", ctypes.c_void_p),
+        ("n", ctypes.c_int64),
+        ("k", ctypes.c_int64),
+        ("g", ctypes.c_int32),
+        ("y_dtype", ctypes.c_int32),
+    ]
+
+
+def load(path: Optional[str] = None):
+    """Load libtq.so (built by ``paper_2606_18114_gb300.build``) once."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    p = path or _LIB_PATH
+    if not os.path.exists(p):
+        raise RuntimeError(f"libtq.so not found at {p}; run paper_2606_18114_gb300.build.build()")
+    lib = ctypes.CDLL(p)
+    i64, i32, vp = ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p
+    lib.tq_quantize.argtypes = [vp, i64, i64, i32, vp, vp, vp, vp]
+    lib.tq_linear_fwd.argtypes = [vp, i64, i64, vp, vp, i64, i32, vp, i32, vp]
+    lib.tq_linear_bwd.argtypes = [vp, vp, i64, i64, i64, vp, vp, i32, vp, i32, vp, i32, vp]
+    lib.tq_linear_fwd_batched.argtypes = [ctypes.POINTER(FwdDesc), i32, i64, vp]
+    lib.tq_device_status.argtypes = [vp]
+    for name in ("tq_quantize", "tq_linear_fwd", "tq_linear_bwd", "tq_linear_fwd_batched",
+                 "tq_device_status"):
+        getattr(lib, name).restype = ctypes.c_int
+    lib.tq_last_error.restype = ctypes.c_char_p
+    lib.tq_last_error.argtypes = []
+    lib.tq_version.restype = ctypes.c_char_p
+    lib.tq_version.argtypes = []
+    _lib = lib
+    return lib
+
+
+def _check(status: int):
+    if status != 0:
+        raise TqError(status, load().tq_last_error().decode())
+
+
+def _stream(stream=None) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream)
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    if t is None:
+        return None
+    if not t.is_contiguous():
+        raise ValueError("tensors passed to libtq must be contiguous")
+    return t.data_ptr() or None
+
+
+def version() -> str:
+    return load().tq_version().decode()
+
+
+def device_status(stream=None) -> None:
+    """Synchronise the stream and raise if a kernel's bounded wait ran out."""
+    _check(load().tq_device_status(_stream(stream)))
+
+
+def quantize(w: torch.Tensor, g: int, out=None, stream=None):
+    """§3.1 quantiser on a CUDA fp32 ``w [N, K]``.
+
+    Returns ``(codes uint32-as-int32 [N, K/16], scales fp32 [N, K/g],
+    zero_counts int32 [N, K/g])``. ``codes`` is an int32 tensor holding the
+    uint32 bit patterns.
+    """
+    n, k = w.shape
+    if out is None:
+        codes = torch.empty((n, k // 16), dtype=torch.int32, device=w.device)
+        scales = torch.empty((n, k // g), dtype=torch.float32, device=w.device)
+        zeros = torch.empty((n, k // g), dtype=torch.int32, device=w.device)
+    else:
+        codes, scales, zeros = out
+    _check(load().tq_quantize(_ptr(w), n, k, g, _ptr(codes), _ptr(scales), _ptr(zeros),
+                              _stream(stream)))
+    return codes, scales, zeros
+
+
+def _out_code(dtype) -> int:
+    if dtype == torch.float32:
+        return OUT_F32
+    if dtype == torch.bfloat16:
+        return OUT_BF16
+    raise ValueError(f"unsupported output dtype {dtype}")
+
+
+def linear_fwd(x: torch.Tensor, codes: torch.Tensor, scales: torch.Tensor, g: int,
+               out_dtype=torch.float32, y: Optional[torch.Tensor] = None, stream=None):
+    """W1.58A16 forward ``y = x W^T`` for bf16 ``x [M, K]``; returns ``y [M, N]``."""
+    m, k = x.shape
+    n = codes.shape[0]
+    if y is None:
+        y = torch.empty((m, n), dtype=out_dtype, device=x.device)
+    _check(load().tq_linear_fwd(_ptr(x), m, k, _ptr(codes), _ptr(scales), n, g, _ptr(y),
+                                _out_code(y.dtype), _stream(stream)))
+    return y
+
+
+def linear_bwd(dy: torch.Tensor, x: Optional[torch.Tensor], codes: torch.Tensor,
+               scales: torch.Tensor, k: int, g: int, want_dx: bool = True, want_dw: bool = True,
+               dx_dtype=torch.float32, dx: Optional[torch.Tensor] = None,
+               dw: Optional[torch.Tensor] = None, accumulate_dw: bool = False, stream=None):
+    """STE backward; returns ``(dx [M, K] or None, dw fp32 [N, K] or None)``."""
+    m, n = dy.shape
+    if want_dx and dx is None:
+        dx = torch.empty((m, k), dtype=dx_dtype, device=dy.device)
+    if want_dw and dw is None:
+        dw = torch.empty((n, k), dtype=torch.float32, device=dy.device)
+    if not want_dx:
+        dx = None
+    if not want_dw:
+        dw = None
+    _check(load().tq_linear_bwd(_ptr(dy), _ptr(x), m, n, k, _ptr(codes), _ptr(scales), g,
+                                _ptr(dx), _out_code(dx.dtype) if dx is not None else OUT_F32,
+                                _ptr(dw), int(accumulate_dw), _stream(stream)))
+    return dx, dw
+
+
+def linear_fwd_batched(items: Sequence[dict], m: int, stream=None) -> None:
+    """Decode forward over many matrices in one call.
+
+    ``items``: dicts with ``x, codes, scales, y, g`` (tensors already allocated,
+    ``y`` written in place).
+    """
+    arr = (FwdDesc * len(items))()
+    for i, it in enumerate(items):
+        codes = it["codes"]
+        arr[i] = FwdDesc(_ptr(it["x"]), _ptr(codes), _ptr(it["scales"]), _ptr(it["y"]),
+                         codes.shape[0], codes.shape[1] * 16, it["g"], _out_code(it["y"].dtype))
+    _check(load().tq_linear_fwd_batched(arr, len(items), m, _stream(stream)))

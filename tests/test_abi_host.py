@@ -1,0 +1,119 @@
+"""Host-side checks of the C ABI (no GPU): the library loads, exports every
+symbol include/tq.h declares, and rejects bad arguments before touching a device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2606_18114_gb300 import build as tqbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    path = tqbuild.build()
+    from paper_2606_18114_gb300 import tq
+    return tq.load(path)
+
+
+def _declared():
+    with open(os.path.join(ROOT, "include", "tq.h")) as f:
+        text = f.read()
+    return re.findall(r"TQ_API\s+[\w\s\*]+?\b(tq_\w+)\s*\(", text)
+
+
+def test_header_declares_expected_symbols():
+    from paper_2606_18114_gb300 import tq
+    assert sorted(_declared()) == sorted(tq.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in _declared():
+        assert hasattr(lib, name), name
+
+
+def test_exports_are_exactly_the_header(lib):
+    import subprocess
+    out = subprocess.run(["nm", "-D", "--defined-only", lib._name], capture_output=True, text=True)
+    if out.returncode != 0:
+        pytest.skip("nm unavailable")
+    tq_syms = sorted(set(re.findall(r"\b(tq_\w+)\b", out.stdout)))
+    assert tq_syms == sorted(_declared())
+
+
+def test_version_and_empty_error(lib):
+    assert b"sm_103a" in lib.tq_version()
+    assert lib.tq_last_error() is not None
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    from paper_2606_18114_gb300 import tq
+    saved = tq._lib
+    tq._lib = None
+    try:
+        with pytest.raises(RuntimeError):
+            tq.load(str(tmp_path / "nope.so"))
+    finally:
+        tq._lib = saved
+
+
+FAKE = 1 << 20  # aligned, never dereferenced: every call below fails validation first
+MIS = FAKE + 4  # misaligned
+
+
+@pytest.mark.parametrize("args,status", [
+    ((FAKE, 8, 256, 33, FAKE, FAKE, FAKE, None), 1),   # bad group size
+    ((FAKE, 8, 200, 32, FAKE, FAKE, FAKE, None), 1),   # k % 16
+    ((FAKE, 8, 96, 64, FAKE, FAKE, FAKE, None), 1),    # k % g
+    ((FAKE, -1, 256, 32, FAKE, FAKE, FAKE, None), 1),  # negative
+    ((None, 8, 256, 32, FAKE, FAKE, FAKE, None), 1),   # null w
+    ((MIS, 8, 256, 32, FAKE, FAKE, FAKE, None), 1),    # misaligned w
+    ((FAKE, 8, 256, 32, FAKE, None, FAKE, None), 1),   # null scales
+    ((None, 0, 256, 32, None, None, None, None), 0),   # empty: nothing to do
+    ((None, 8, 0, 32, None, None, None, None), 0),
+])
+def test_quantize_rejects_before_launch(lib, args, status):
+    assert lib.tq_quantize(*args) == status
+    if status:
+        assert lib.tq_last_error()
+
+
+@pytest.mark.parametrize("args,status", [
+    ((FAKE, 4, 256, FAKE, FAKE, 64, 48, FAKE, 0, None), 1),    # bad group
+    ((FAKE, 4, 96, FAKE, FAKE, 64, 32, FAKE, 0, None), 2),     # k % 64 unsupported
+    ((FAKE, 4, 256, FAKE, FAKE, 64, 512, FAKE, 0, None), 1),   # k % g
+    ((FAKE, 4, 256, FAKE, FAKE, 64, 32, FAKE, 7, None), 1),    # bad dtype
+    ((None, 4, 256, FAKE, FAKE, 64, 32, FAKE, 0, None), 1),    # null x
+    ((FAKE, 4, 256, MIS, FAKE, 64, 32, FAKE, 0, None), 1),     # misaligned codes
+    ((FAKE, 4, 256, FAKE, FAKE, 64, 32, None, 0, None), 1),    # null y
+    ((None, 0, 256, None, None, 64, 32, None, 0, None), 0),    # m = 0
+    ((None, 4, 256, None, None, 0, 32, None, 0, None), 0),     # n = 0
+])
+def test_linear_fwd_rejects_before_launch(lib, args, status):
+    assert lib.tq_linear_fwd(*args) == status
+
+
+@pytest.mark.parametrize("args,status", [
+    ((FAKE, FAKE, 4, 60, 256, FAKE, FAKE, 32, FAKE, 0, FAKE, 0, None), 2),  # n % 8
+    ((FAKE, FAKE, 4, 64, 256, FAKE, FAKE, 32, None, 0, None, 0, None), 1),  # no output
+    ((FAKE, None, 4, 64, 256, FAKE, FAKE, 32, None, 0, FAKE, 0, None), 1),  # dw needs x
+    ((None, FAKE, 4, 64, 256, FAKE, FAKE, 32, FAKE, 0, None, 0, None), 1),  # dx needs dy
+    ((FAKE, FAKE, 4, 64, 256, FAKE, FAKE, 32, FAKE, 3, None, 0, None), 1),  # bad dtype
+    ((FAKE, FAKE, 4, 64, 256, None, FAKE, 32, FAKE, 0, None, 0, None), 1),  # dx needs codes
+])
+def test_linear_bwd_rejects_before_launch(lib, args, status):
+    assert lib.tq_linear_bwd(*args) == status
+
+
+def test_batched_rejects_before_launch(lib):
+    from paper_2606_18114_gb300.tq import FwdDesc
+    arr = (FwdDesc * 2)()
+    arr[0] = FwdDesc(FAKE, FAKE, FAKE, FAKE, 64, 256, 32, 0)
+    arr[1] = FwdDesc(FAKE, FAKE, FAKE, FAKE, 64, 250, 32, 0)  # k % g
+    assert lib.tq_linear_fwd_batched(arr, 2, 1, None) == 1
+    assert b"descs[1]" in lib.tq_last_error()
+    assert lib.tq_linear_fwd_batched(arr, 1, 17, None) == 1   # m > 16
+    assert lib.tq_linear_fwd_batched(arr, 300, 1, None) == 1  # count > max
+    assert lib.tq_linear_fwd_batched(None, 0, 1, None) == 0   # nothing to do

@@ -1,0 +1,222 @@
+"""CUDA path vs oracle, element by element, through the C ABI (needs a GB300).
+
+Inputs come from ``paper_2606_18114_gb300.synth`` (seeded, host-side); the
+oracle never sees a value produced by the CUDA path.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import tq_oracle as O
+from paper_2606_18114_gb300 import synth
+from parity import check_close, check_quantize, codes_u32, to_np
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def tq():
+    if not torch.cuda.is_available():
+        pytest.fail("the gpu tests need a CUDA device")
+    from paper_2606_18114_gb300 import build, tq as _tq
+    build.build()
+    _tq.load()
+    return _tq
+
+
+def _quant(tq, w_np, g):
+    w = torch.from_numpy(w_np).cuda()
+    codes, s, z = tq.quantize(w, g)
+    tq.device_status()
+    return codes, s, z
+
+
+# ------------------------------------------------------------------ quantize
+def test_quantize_hand_example_g128(tq, golden_dir):
+    import json, os
+    with open(os.path.join(golden_dir, "hand_2group.json")) as f:
+        gd = json.load(f)
+    w = np.repeat(np.array(gd["w"], dtype=np.float32).reshape(2, 4), 32, axis=1).reshape(1, 256)
+    codes, s, z = _quant(tq, w, 128)
+    assert to_np(s)[0].tolist() == gd["g128_embedding"]["scales"]
+    assert to_np(z)[0].tolist() == gd["g128_embedding"]["zero_counts"]
+    c = O.unpack(codes_u32(codes), 256)[0]
+    assert c.reshape(2, 4, 32)[:, :, 0].reshape(-1).tolist() == gd["codes"]
+
+
+def test_quantize_exact_tie_goes_to_zero(tq):
+    # |w/s| = 0.5 exactly: round half to even gives 0 (tie reading of §3.1).
+    w = np.tile(np.array([0.25, 0.75, 1.0, 0.0], dtype=np.float32), 8).reshape(1, 32)
+    w = np.concatenate([w, -w], axis=0)
+    codes, s, z = _quant(tq, w, 32)
+    assert to_np(s).tolist() == [[0.5], [0.5]]
+    c = O.unpack(codes_u32(codes), 32)
+    assert c[0, :4].tolist() == [0, 1, 1, 0] and c[1, :4].tolist() == [0, -1, -1, 0]
+    assert to_np(z).tolist() == [[16], [16]]
+
+
+def test_quantize_zero_groups(tq):
+    w = synth.latent_weights(4, 512, seed=1)
+    w[1] = 0.0
+    w[2, 128:256] = 0.0
+    codes, s, z = _quant(tq, w, 128)
+    check_quantize(w, 128, codes, s, z)
+    assert to_np(z)[1].tolist() == [128] * 4 and to_np(s)[1].tolist() == [0.0] * 4
+
+
+@pytest.mark.parametrize("n,k,g", [
+    (512, 256, 128),   # single grouped ternary linear
+    (7, 96, 32),       # partial warp unit
+    (33, 320, 64),
+    (3, 768, 256),     # half of the last unit
+    (5, 1536, 512),
+    (1, 32, 32),
+    (1, 16 * 3 * 32, 32),
+])
+def test_quantize_shapes(tq, n, k, g):
+    w = synth.latent_weights(n, k, seed=n + k + g)
+    codes, s, z = _quant(tq, w, g)
+    check_quantize(w, g, codes, s, z)
+
+
+@pytest.mark.parametrize("g", [32, 64, 128, 256, 512])
+@pytest.mark.parametrize("dist", ["gauss", "t3"])
+def test_quantize_group_sizes(tq, g, dist):
+    w = synth.latent_weights(96, 2048, seed=g, dist=dist)
+    codes, s, z = _quant(tq, w, g)
+    check_quantize(w, g, codes, s, z)
+
+
+def test_quantize_scaled_values(tq):
+    w = synth.latent_weights(64, 1024, seed=9) * np.float32(2.0 ** 20)
+    codes, s, z = _quant(tq, w, 128)
+    check_quantize(w, 128, codes, s, z)
+
+
+@pytest.mark.parametrize("proj", ["in_proj", "out_proj"])
+@pytest.mark.parametrize("dist", ["gauss", "t3"])
+def test_quantize_mamba2_full(tq, proj, dist):
+    n, k = synth.MAMBA2_1P3B[proj]
+    w = synth.latent_weights(n, k, seed=0, dist=dist)
+    codes, s, z = _quant(tq, w, 128)
+    flips, ties = check_quantize(w, 128, codes, s, z)
+    assert flips <= ties
+    ratio = to_np(z).sum() / w.size
+    assert (0.30 < ratio < 0.32) if dist == "gauss" else (0.36 < ratio < 0.39)
+
+
+# ------------------------------------------------------------------ linear
+def _setup(tq, n, k, m, g, seed=0, dy_std=1.0, dist="gauss"):
+    w = synth.latent_weights(n, k, seed=seed, dist=dist)
+    x = synth.activations_bf16(m, k, seed=seed, stream="x")
+    dy = synth.activations_bf16(m, n, seed=seed, std=dy_std, stream="dy")
+    ref = O.quantize(w, g)
+    w_hat = O.dequantize(ref[0], ref[1], k, g)
+    codes, s, z = _quant(tq, w, g)
+    return w, x, dy, w_hat, codes, s
+
+
+@pytest.mark.parametrize("n,k,m,g", [
+    (512, 256, 64, 128),     # single grouped ternary linear (seed 0)
+    (200, 192, 300, 64),     # ragged rows, tokens and reduction
+    (136, 320, 257, 32),
+    (264, 512, 17, 256),     # smallest GEMM token count
+    (128, 1024, 256, 512),
+    (520, 1024, 1, 128),     # decode
+    (520, 1024, 3, 128),
+    (520, 1024, 16, 128),
+    (40, 64, 5, 32),         # one k-block
+])
+def test_linear_parity(tq, n, k, m, g):
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=n + k + m)
+    xd, dyd = x.cuda(), dy.cuda()
+    y = tq.linear_fwd(xd, codes, s, g)
+    dx, dw = tq.linear_bwd(dyd, xd, codes, s, k, g)
+    tq.device_status()
+    check_close(y, O.linear_fwd(x, w_hat), "Y")
+    check_close(dx, O.linear_bwd_dx(dy, w_hat), "dX")
+    check_close(dw, O.linear_bwd_dw(dy, x), "dW")
+
+
+def test_linear_bf16_outputs_are_rounded_fp32(tq):
+    n, k, m, g = 264, 512, 300, 128
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=3)
+    xd, dyd = x.cuda(), dy.cuda()
+    y32 = tq.linear_fwd(xd, codes, s, g)
+    y16 = tq.linear_fwd(xd, codes, s, g, out_dtype=torch.bfloat16)
+    dx32, _ = tq.linear_bwd(dyd, xd, codes, s, k, g, want_dw=False)
+    dx16, _ = tq.linear_bwd(dyd, xd, codes, s, k, g, want_dw=False, dx_dtype=torch.bfloat16)
+    tq.device_status()
+    assert torch.equal(y16, y32.to(torch.bfloat16))
+    assert torch.equal(dx16, dx32.to(torch.bfloat16))
+    check_close(y16, O.linear_fwd(x, w_hat), "Y bf16", max_rel_rms=3e-2)
+
+
+def test_dw_accumulate_and_single_outputs(tq):
+    n, k, m, g = 136, 256, 200, 64
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=4)
+    xd, dyd = x.cuda(), dy.cuda()
+    base = torch.randn(n, k, device="cuda", dtype=torch.float32)
+    base_np = to_np(base).astype(np.float64)
+    dw = base.clone()
+    dx, dw = tq.linear_bwd(dyd, xd, codes, s, k, g, want_dx=False, dw=dw, accumulate_dw=True)
+    assert dx is None
+    dx2, dw2 = tq.linear_bwd(dyd, None, codes, s, k, g, want_dw=False)
+    tq.device_status()
+    assert dw2 is None
+    check_close(to_np(dw) - base_np, O.linear_bwd_dw(dy, x), "dW accumulated")
+    check_close(dx2, O.linear_bwd_dx(dy, w_hat), "dX only")
+
+
+def test_empty_sizes(tq):
+    codes = torch.zeros((64, 256 // 16), dtype=torch.int32, device="cuda")
+    s = torch.zeros((64, 2), dtype=torch.float32, device="cuda")
+    x = torch.zeros((0, 256), dtype=torch.bfloat16, device="cuda")
+    y = tq.linear_fwd(x, codes, s, 128)
+    assert y.shape == (0, 64)
+    dy = torch.zeros((0, 64), dtype=torch.bfloat16, device="cuda")
+    dw = torch.full((64, 256), 7.0, device="cuda")
+    tq.linear_bwd(dy, x, codes, s, 256, 128, want_dx=False, dw=dw)
+    tq.device_status()
+    assert float(dw.abs().max()) == 0.0   # M = 0: dW = empty sum = 0
+
+
+def test_batched_decode_matches_single(tq):
+    mats = []
+    for i, (n, k) in enumerate([(520, 256), (256, 512), (520, 256), (136, 1024)]):
+        w = synth.latent_weights(n, k, seed=100 + i)
+        x = synth.activations_bf16(4, k, seed=100 + i)
+        codes, s, _ = _quant(tq, w, 128)
+        ref = O.quantize(w, 128)
+        w_hat = O.dequantize(ref[0], ref[1], k, 128)
+        mats.append(dict(x=x.cuda(), codes=codes, scales=s, g=128,
+                         y=torch.empty((4, n), device="cuda"), ref=O.linear_fwd(x, w_hat)))
+    tq.linear_fwd_batched(mats, 4)
+    tq.device_status()
+    for i, it in enumerate(mats):
+        check_close(it["y"], it["ref"], f"batched Y[{i}]")
+
+
+# ------------------------------------------------------------------ full size
+@pytest.mark.parametrize("proj", ["in_proj", "out_proj"])
+def test_linear_mamba2_prefill_sampled(tq, proj):
+    """Full Mamba-2 1.3B projection at batch 8 x seq 2048, checked on sampled rows."""
+    n, k = synth.MAMBA2_1P3B[proj]
+    m, g = 16384, 128
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=0, dy_std=1e-2)
+    xd, dyd = x.cuda(), dy.cuda()
+    y = tq.linear_fwd(xd, codes, s, g)
+    dx, dw = tq.linear_bwd(dyd, xd, codes, s, k, g)
+    tq.device_status()
+    rs = np.random.default_rng(1)
+    rows = np.sort(rs.choice(m, 64, replace=False))
+    nrows = np.sort(rs.choice(n, 64, replace=False))
+    check_close(to_np(y[torch.from_numpy(rows).cuda()]), O.linear_fwd(x, w_hat, rows), "Y rows")
+    check_close(to_np(dx[torch.from_numpy(rows).cuda()]), O.linear_bwd_dx(dy, w_hat, rows),
+                "dX rows")
+    check_close(to_np(dw[torch.from_numpy(nrows).cuda()]), O.linear_bwd_dw(dy, x, nrows),
+                "dW rows")
+    # every output finite, and the sampled tail rows of the ragged N tile too
+    assert torch.isfinite(y).all() and torch.isfinite(dx).all() and torch.isfinite(dw).all()
+    tail = np.arange(n - 8, n)
+    check_close(to_np(dw[torch.from_numpy(tail).cuda()]), O.linear_bwd_dw(dy, x, tail), "dW tail")
