@@ -404,6 +404,40 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_only(args):
+    """One kernel of the step in isolation (for ncu captures of a single launch)."""
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_18114_gb300 import tq
+    torch.cuda.set_device(0)
+    if args.only == "decode":
+        res = decode_sweep(tq, (1,), args.steps, args.warmup)
+        print(json.dumps({"only": "decode", **res}), flush=True)
+        return
+    p = Prefill(tq, IN_PROJ[0], IN_PROJ[1], M_PREFILL, G, seed=7)
+    tq.quantize(p.w, p.g, out=(p.codes, p.s, p.z))
+    calls = {
+        "quantize": lambda: tq.quantize(p.w, p.g, out=(p.codes, p.s, p.z)),
+        "fwd": lambda: tq.linear_fwd(p.x, p.codes, p.s, p.g, y=p.y),
+        "dx": lambda: tq.linear_bwd(p.dy, p.x, p.codes, p.s, p.k, p.g, want_dw=False, dx=p.dx),
+        "dw": lambda: tq.linear_bwd(p.dy, p.x, p.codes, p.s, p.k, p.g, want_dx=False, dw=p.dw),
+    }
+    fn = calls[args.only]
+    for _ in range(args.warmup):
+        fn()
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(args.steps):
+        fn()
+    t1.record()
+    torch.cuda.synchronize()
+    tq.device_status()
+    print(json.dumps({"only": args.only, "ms": t0.elapsed_time(t1) / max(args.steps, 1)}),
+          flush=True)
+
+
 # ------------------------------------------------------------------ main
 def main():
     ap = argparse.ArgumentParser()
@@ -413,9 +447,15 @@ def main():
     ap.add_argument("--impl", default="tq", choices=["tq", "reference"])
     ap.add_argument("--no-extra", action="store_true", help="skip decode/quantize sweeps")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
+    ap.add_argument("--only", choices=["quantize", "fwd", "dx", "dw", "decode"],
+                    help="profiling aid: run just this kernel of the step (or the batched "
+                         "M=1 decode) --warmup + --steps times and print its time")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)
+        return
+    if args.only:
+        run_only(args)
         return
     if args.warmup < 3:
         args.warmup = 3

@@ -2,17 +2,22 @@
 // estimator hands the gradient of the dequantised weight to the latent fp32 W
 // unchanged). A plain bf16 x bf16 -> fp32 tcgen05 GEMM; quantisation plays no part.
 //
-// Tile: 128 input features k (TMEM lanes) x 256 output features n (TMEM columns);
-// the reduction runs over the tokens m, which is the outer (row) dimension of both
-// x [m][k] and dy [m][n], so both operands are MN-major. Each 64-token k-block
-// is TMA-loaded as boxes of 64 features x 64 tokens with the 128-byte swizzle:
-// two boxes for x (A, 128 features) and four for dy (B, 256 features). In the
-// canonical MN-major layout the leading byte offset is the distance between
+// Output tile: 128 input features k (TMEM lanes) x 256 output features n (TMEM
+// columns). The reduction runs over the tokens m, the outer (row) dimension of
+// both x [m][k] and dy [m][n], so both operands are MN-major. Each 64-token
+// k-block is TMA-loaded as boxes of 64 features x 64 tokens with the 128-byte
+// swizzle: two boxes for x (A, 128 features) and four for dy (B, 256 features).
+// In the canonical MN-major layout the leading byte offset is the distance between
 // 64-feature chunks (one box, 8 KB) and the stride byte offset the distance
 // between groups of 8 tokens (1 KB).
 //
-// The epilogue thread of lane k writes dW[n][k] for the tile's columns n, so a
-// warp's store covers 32 consecutive k of one row n (128 contiguous bytes).
+// Persistent: one CTA per SM walks the tiles, k-tiles fastest, so that the CTAs in
+// flight stream the same dy columns. x is loaded with an L2 evict-last policy (it
+// is re-read by every n-tile and fits in L2), dy with evict-first. Two TMEM
+// accumulators (2 x 256 columns) let the epilogue of one tile overlap the main loop
+// of the next. Roles: warp 0 TMA, warp 1 MMA, warps 2-5 epilogue; the epilogue
+// thread of lane k writes dW[n][k], so a warp store covers 32 consecutive k of
+// one row n (128 contiguous bytes).
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -30,8 +35,31 @@ constexpr int kABytes = 2 * kBox;   // 128 features
 constexpr int kBBytes = 4 * kBox;   // 256 features
 constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kBarOff = kStages * kStageBytes;
-constexpr int kBytes = kBarOff + (2 * kStages + 1) * 8 + 8;
-constexpr uint32_t kTmemCols = 256;
+constexpr int kNumBars = 2 * kStages + 4;
+constexpr int kBytes = kBarOff + kNumBars * 8 + 8;
+constexpr uint32_t kTmemCols = 512;
+
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap* map,
+                                                 uint32_t bar, int32_t x, int32_t y,
+                                                 uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(policy)
+      : "memory");
+}
 
 __global__ void __launch_bounds__(kThreads, 1)
     dw_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x,
@@ -41,24 +69,37 @@ __global__ void __launch_bounds__(kThreads, 1)
                                              ~static_cast<uintptr_t>(1023));
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int64_t k0 = static_cast<int64_t>(blockIdx.x) * kDwTileK;
-  const int64_t n0 = static_cast<int64_t>(blockIdx.y) * kDwTileN;
   const int nkb = static_cast<int>((args.m + kKBlock - 1) / kKBlock);
+  const uint32_t k_tiles = static_cast<uint32_t>((args.k + kDwTileK - 1) / kDwTileK);
+  const uint32_t tiles = k_tiles * static_cast<uint32_t>((args.n + kDwTileN - 1) / kDwTileN);
+  const int my_tiles =
+      blockIdx.x < tiles ? static_cast<int>((tiles - 1 - blockIdx.x) / gridDim.x + 1) : 0;
+  const int total = my_tiles * nkb;
   int* status = args.status;
+  auto tile_k0 = [&](int i) -> int64_t {
+    return static_cast<int64_t>((blockIdx.x + static_cast<uint32_t>(i) * gridDim.x) % k_tiles) * kDwTileK;
+  };
+  auto tile_n0 = [&](int i) -> int64_t {
+    return static_cast<int64_t>((blockIdx.x + static_cast<uint32_t>(i) * gridDim.x) / k_tiles) * kDwTileN;
+  };
 
   const uint32_t smem_base = smem_u32(smem);
   const uint32_t bar_base = smem_base + kBarOff;
   auto full_bar = [&](int s) { return bar_base + 8u * s; };
   auto empty_bar = [&](int s) { return bar_base + 8u * (kStages + s); };
-  const uint32_t acc_bar = bar_base + 8u * (2 * kStages);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kBarOff + (2 * kStages + 1) * 8);
+  auto accfull_bar = [&](int a) { return bar_base + 8u * (2 * kStages + a); };
+  auto accempty_bar = [&](int a) { return bar_base + 8u * (2 * kStages + 2 + a); };
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kBarOff + kNumBars * 8);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(full_bar(s), 1);
       mbar_init(empty_bar(s), 1);
     }
-    mbar_init(acc_bar, 1);
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(accfull_bar(a), 1);
+      mbar_init(accempty_bar(a), 128);
+    }
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -72,78 +113,99 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem_acc = *tmem_slot;
+  const uint32_t tmem_base = *tmem_slot;
 
   if (warp == 0) {
     if (lane == 0) {
+      const uint64_t keep = policy_evict_last();
+      const uint64_t stream = policy_evict_first();
       int issued = 0;
       bool ok = true;
-      for (int kb = 0; kb < nkb; ++kb) {
-        const int s = kb % kStages;
-        const uint32_t ph = (kb / kStages) & 1;
+      for (int it = 0; it < total; ++it) {
+        const int i = it / nkb, kb = it - i * nkb;
+        const int s = it % kStages;
+        const uint32_t ph = (it / kStages) & 1;
         if (!(ok = mbar_wait(empty_bar(s), ph ^ 1, status))) break;
         const uint32_t a = smem_base + s * kStageBytes;
         const uint32_t b = a + kABytes;
         const int32_t mrow = kb * kKBlock;
+        const int64_t k0 = tile_k0(i), n0 = tile_n0(i);
         mbar_arrive_expect_tx(full_bar(s), kStageBytes);
 #pragma unroll
         for (int c = 0; c < 2; ++c)
-          tma_load_2d(a + c * kBox, &tmap_x, full_bar(s), static_cast<int32_t>(k0 + 64 * c), mrow);
+          tma_load_2d_hint(a + c * kBox, &tmap_x, full_bar(s), static_cast<int32_t>(k0 + 64 * c),
+                           mrow, keep);
 #pragma unroll
         for (int c = 0; c < 4; ++c)
-          tma_load_2d(b + c * kBox, &tmap_dy, full_bar(s), static_cast<int32_t>(n0 + 64 * c), mrow);
+          tma_load_2d_hint(b + c * kBox, &tmap_dy, full_bar(s), static_cast<int32_t>(n0 + 64 * c),
+                           mrow, stream);
         ++issued;
       }
       if (!ok) {
-        for (int kb = issued - 1; kb >= 0 && kb >= issued - kStages; --kb)
-          mbar_wait(full_bar(kb % kStages), (kb / kStages) & 1, status);
+        for (int it = issued - 1; it >= 0 && it >= issued - kStages; --it)
+          mbar_wait(full_bar(it % kStages), (it / kStages) & 1, status);
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(128, kDwTileN, 1, 1);
-      for (int kb = 0; kb < nkb; ++kb) {
-        const int s = kb % kStages;
-        const uint32_t ph = (kb / kStages) & 1;
-        if (!mbar_wait(full_bar(s), ph, status)) break;
+      int it = 0;
+      bool ok = true;
+      for (int i = 0; i < my_tiles && ok; ++i) {
+        const int acc = i & 1;
+        const uint32_t aph = (i >> 1) & 1;
+        if (!(ok = mbar_wait(accempty_bar(acc), aph ^ 1, status))) break;
         tc_fence_after();
-        const uint32_t a = smem_base + s * kStageBytes;
-        const uint32_t b = a + kABytes;
+        const uint32_t d = tmem_base + acc * kDwTileN;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = it % kStages;
+          const uint32_t ph = (it / kStages) & 1;
+          if (!(ok = mbar_wait(full_bar(s), ph, status))) break;
+          tc_fence_after();
+          const uint32_t a = smem_base + s * kStageBytes;
+          const uint32_t b = a + kABytes;
 #pragma unroll
-        for (int j = 0; j < kKBlock / 16; ++j) {
-          // 16 tokens = two 8-token core groups = 2 KB further into each box
-          const uint64_t adesc = smem_desc_sw128(a + j * 2048, kBox, 1024);
-          const uint64_t bdesc = smem_desc_sw128(b + j * 2048, kBox, 1024);
-          mma_ss(tmem_acc, adesc, bdesc, idesc, (kb | j) != 0);
+          for (int j = 0; j < kKBlock / 16; ++j) {
+            // 16 tokens = two 8-token core groups = 2 KB further into each box
+            const uint64_t adesc = smem_desc_sw128(a + j * 2048, kBox, 1024);
+            const uint64_t bdesc = smem_desc_sw128(b + j * 2048, kBox, 1024);
+            mma_ss(d, adesc, bdesc, idesc, (kb | j) != 0);
+          }
+          mma_commit(empty_bar(s));
         }
-        mma_commit(empty_bar(s));
+        if (ok) mma_commit(accfull_bar(acc));
       }
-      mma_commit(acc_bar);
     }
   } else {
     const int quad = warp & 3;
-    const int64_t kk = k0 + quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
-    const bool ok = __all_sync(0xffffffffu, mbar_wait(acc_bar, 0, status));
-    tc_fence_after();
-    if (ok) {
+    for (int i = 0; i < my_tiles; ++i) {
+      const int acc = i & 1;
+      const uint32_t aph = (i >> 1) & 1;
+      if (!__all_sync(0xffffffffu, mbar_wait(accfull_bar(acc), aph, status))) break;
+      tc_fence_after();
+      const int64_t kk = tile_k0(i) + quad * 32 + lane;
+      const int64_t n0 = tile_n0(i);
+      const uint32_t d = tmem_base + acc * kDwTileN + lane_off;
 #pragma unroll 1
-      for (int c = 0; c < kDwTileN; c += 32) {
-        uint32_t v[32];
-        tmem_ld_x32(tmem_acc + lane_off + c, v);
-        tmem_ld_wait(v);
+      for (int c = 0; c < kDwTileN; c += 16) {
+        uint32_t v[16];
+        tmem_ld16(d + c, v);
+        tmem_ld_wait16(v);
         if (kk < args.k) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int64_t n = n0 + c + i;
+          for (int t = 0; t < 16; ++t) {
+            const int64_t n = n0 + c + t;
             if (n < args.n) {
               float* p = args.dw + n * args.k + kk;
-              const float val = __uint_as_float(v[i]);
+              const float val = __uint_as_float(v[t]);
               *p = args.accumulate ? *p + val : val;
             }
           }
         }
       }
+      tc_fence_before();
+      mbar_arrive(accempty_bar(acc));
     }
   }
 
@@ -152,7 +214,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem_acc, kTmemCols);
+    tmem_dealloc(tmem_base, kTmemCols);
   }
 }
 
@@ -161,14 +223,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 size_t dw_smem_bytes() { return kBytes + 1024; }
 
 cudaError_t launch_dw_gemm(const CUtensorMap& tmap_x, const CUtensorMap& tmap_dy,
-                           const DwArgs& a, cudaStream_t stream) {
+                           const DwArgs& a, int num_sms, cudaStream_t stream) {
   const size_t smem = dw_smem_bytes();
   cudaError_t e = cudaFuncSetAttribute(dw_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  dim3 grid(static_cast<unsigned>((a.k + kDwTileK - 1) / kDwTileK),
-            static_cast<unsigned>((a.n + kDwTileN - 1) / kDwTileN));
-  dw_gemm_kernel<<<grid, kThreads, smem, stream>>>(tmap_x, tmap_dy, a);
+  const int64_t tiles = ((a.k + kDwTileK - 1) / kDwTileK) * ((a.n + kDwTileN - 1) / kDwTileN);
+  const int64_t grid = tiles < num_sms ? tiles : num_sms;
+  dw_gemm_kernel<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(tmap_x, tmap_dy, a);
   return cudaGetLastError();
 }
 

@@ -30,12 +30,12 @@ struct TsArgs {
 
 // Tile of the activation operand along the token dimension.
 int ts_tile_tokens(int64_t m);
-size_t ts_smem_bytes(int bn);
 
 // tmap_b: bf16 activations [m][red] with box {64, bn}, 128-byte swizzle.
 // tmap_codes: uint32 codes [wn][wk/16] with box {4, 128} (fwd) or {8, 64} (dx).
+// Persistent: min(tiles, num_sms) CTAs.
 cudaError_t launch_ts_gemm(int mode, int bn, const CUtensorMap& tmap_b,
-                           const CUtensorMap& tmap_codes, const TsArgs& args,
+                           const CUtensorMap& tmap_codes, const TsArgs& args, int num_sms,
                            cudaStream_t stream);
 
 // dw_gemm.cu -----------------------------------------------------------------
@@ -52,8 +52,8 @@ constexpr int kDwTileN = 256;  // columns: output features
 size_t dw_smem_bytes();
 
 // tmap_x: bf16 x [m][k] box {64, 64}; tmap_dy: bf16 dy [m][n] box {64, 64};
-// both with the 128-byte swizzle.
+// both with the 128-byte swizzle. Persistent: min(tiles, num_sms) CTAs.
 cudaError_t launch_dw_gemm(const CUtensorMap& tmap_x, const CUtensorMap& tmap_dy,
-                           const DwArgs& args, cudaStream_t stream);
+                           const DwArgs& args, int num_sms, cudaStream_t stream);
 
 }  // namespace tq

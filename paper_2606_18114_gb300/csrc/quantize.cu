@@ -3,11 +3,20 @@
 //
 // The weight matrix is treated as one flat array: groups (g | k) and code words
 // (16 | k) never straddle a row, so group j of row n is flat group n*(k/g)+j and
-// the outputs are flat arrays too. One warp owns a unit of 512 consecutive
-// weights: four coalesced 16-byte loads per lane, issued before any use. A group
-// is reduced with warp shuffles over the g/4 lanes that hold it (g <= 128), or
-// over the whole warp and several loads (g = 256, 512). The 32 code words of a
-// unit are gathered into lane order and written with one 128-byte store.
+// the outputs are flat arrays too. Each lane owns 16 consecutive weights — one
+// code word — read as four 16-byte loads; a warp covers 512 weights per unit and
+// keeps two units of loads in flight. A group spans g/16 consecutive lanes and is
+// reduced with log2(g/16) xor-shuffles; the zero count of a word is
+// 16 - popc(word & 0x5555...) because every non-zero code has its low bit set.
+//
+// Code decision. The code is +-1 iff fl32(|w| / s) > 0.5 (round half to even sends
+// 0.5 to 0; the clip maps everything beyond 1.5 to +-1). The fp32 quotient exceeds
+// 0.5 exactly when the real quotient exceeds the midpoint 0.5 + 2^-25 between 0.5
+// and its successor, i.e. when |w| - s/2 > s * 2^-25. For s >= 2^-100 both s/2
+// and s * 2^-25 are exact, and |w| - s/2 is exact whenever s/4 <= |w| <= s
+// (Sterbenz); outside that band its rounded value still has the right side of
+// the threshold. So one fused multiply-add and one compare reproduce the
+// correctly rounded division bit for bit. Smaller scales take the division.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -16,14 +25,14 @@
 namespace tq {
 namespace {
 
-constexpr int kUnit = 512;  // weights per warp per iteration
+constexpr int kUnit = 512;    // weights per warp per unit
+constexpr int kUnroll = 2;    // units per warp iteration (loads in flight)
 constexpr int kThreads = 256;
 
-__device__ __forceinline__ uint32_t ternary_code(float w, float s) {
-  // Code +-1 iff |fl32(w / s)| > 0.5 (round half to even sends 0.5 to 0 and the
-  // clip maps everything beyond 1.5 to +-1). s = 0 gives NaN, hence code 0.
-  const float q = __fdiv_rn(w, s);
-  return fabsf(q) > 0.5f ? (q < 0.0f ? 3u : 1u) : 0u;
+__device__ __forceinline__ uint32_t code_bits(float w, float s, float t, bool tiny_s) {
+  const bool nz = tiny_s ? fabsf(__fdiv_rn(w, s)) > 0.5f : __fmaf_rn(-0.5f, s, fabsf(w)) > t;
+  const uint32_t neg = __float_as_uint(w) >> 31;
+  return nz ? (1u | (neg << 1)) : 0u;
 }
 
 template <int G>
@@ -33,112 +42,54 @@ __global__ void __launch_bounds__(kThreads) quantize_kernel(const float* __restr
                                                             float* __restrict__ scales,
                                                             int32_t* __restrict__ zeros) {
   static_assert(G == 32 || G == 64 || G == 128 || G == 256 || G == 512, "group size");
+  constexpr int kLanesPerGroup = G / 16;
+  constexpr float kInvG = 1.0f / G;  // exact: G is a power of two
   const int lane = threadIdx.x & 31;
   const int64_t warp0 = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * kThreads) >> 5;
   const int64_t nunits = (total + kUnit - 1) / kUnit;
-  constexpr float kInvG = 1.0f / G;  // exact: G is a power of two
 
-  for (int64_t u = warp0; u < nunits; u += nwarps) {
-    const int64_t base = u * kUnit;
-    float4 v[4];
+  for (int64_t u0 = warp0 * kUnroll; u0 < nunits; u0 += nwarps * kUnroll) {
+    float4 v[kUnroll][4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int64_t e = base + j * 128 + lane * 4;
-      v[j] = e < total ? __ldcs(reinterpret_cast<const float4*>(w + e))
-                       : make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int r = 0; r < kUnroll; ++r) {
+      const int64_t e = (u0 + r) * kUnit + lane * 16;
+      const bool in = e < total;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        v[r][j] = in ? __ldg(reinterpret_cast<const float4*>(w + e) + j)
+                     : make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    float part[4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j)
-      part[j] = (fabsf(v[j].x) + fabsf(v[j].y)) + (fabsf(v[j].z) + fabsf(v[j].w));
-
-    // s = (1/g) * sum |w| for the group holding each chunk of this lane.
-    float s[4];
-    if constexpr (G <= 128) {
+    for (int r = 0; r < kUnroll; ++r) {
+      const int64_t e = (u0 + r) * kUnit + lane * 16;
+      float sum = 0.f;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        float t = part[j];
+      for (int j = 0; j < 4; ++j)
+        sum += (fabsf(v[r][j].x) + fabsf(v[r][j].y)) + (fabsf(v[r][j].z) + fabsf(v[r][j].w));
 #pragma unroll
-        for (int off = 1; off < G / 4; off <<= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
-        s[j] = t * kInvG;
-      }
-    } else if constexpr (G == 256) {
-      float t0 = part[0] + part[1], t1 = part[2] + part[3];
+      for (int off = 1; off < kLanesPerGroup; off <<= 1)
+        sum += __shfl_xor_sync(0xffffffffu, sum, off);
+      const float s = sum * kInvG;            // s = (1/g) * sum |w|
+      const float t = s * 0x1p-25f;           // half an ulp of 0.5, in units of s
+      const bool tiny = s < 0x1p-100f;
+      const float x[16] = {v[r][0].x, v[r][0].y, v[r][0].z, v[r][0].w,
+                           v[r][1].x, v[r][1].y, v[r][1].z, v[r][1].w,
+                           v[r][2].x, v[r][2].y, v[r][2].z, v[r][2].w,
+                           v[r][3].x, v[r][3].y, v[r][3].z, v[r][3].w};
+      uint32_t word = 0;
 #pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {
-        t0 += __shfl_xor_sync(0xffffffffu, t0, off);
-        t1 += __shfl_xor_sync(0xffffffffu, t1, off);
-      }
-      s[0] = s[1] = t0 * kInvG;
-      s[2] = s[3] = t1 * kInvG;
-    } else {
-      float t = (part[0] + part[1]) + (part[2] + part[3]);
+      for (int i = 0; i < 16; ++i)  // code i at bit 16*(i&1) + 2*(i>>1)
+        word |= code_bits(x[i], s, t, tiny) << (16 * (i & 1) + 2 * (i >> 1));
+      int zc = 16 - __popc(word & 0x55555555u);
 #pragma unroll
-      for (int off = 1; off < 32; off <<= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
-      s[0] = s[1] = s[2] = s[3] = t * kInvG;
-    }
-
-    // Codes: element i = 4*(lane%4) + e of its 16-code word sits at bit
-    // 16*(e&1) + 4*(lane%4) + 2*(e>>1).
-    uint32_t word[4];
-    int zc[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint32_t c0 = ternary_code(v[j].x, s[j]);
-      const uint32_t c1 = ternary_code(v[j].y, s[j]);
-      const uint32_t c2 = ternary_code(v[j].z, s[j]);
-      const uint32_t c3 = ternary_code(v[j].w, s[j]);
-      uint32_t x = (c0 | (c2 << 2) | (c1 << 16) | (c3 << 18)) << (4 * (lane & 3));
-      x |= __shfl_xor_sync(0xffffffffu, x, 1);
-      x |= __shfl_xor_sync(0xffffffffu, x, 2);
-      word[j] = x;
-      zc[j] = (c0 == 0) + (c1 == 0) + (c2 == 0) + (c3 == 0);
-    }
-    // Gather: lane t stores word t of the unit (chunk t/8, lane group t%8).
-    uint32_t mine = 0;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const uint32_t x = __shfl_sync(0xffffffffu, word[j], 4 * (lane & 7));
-      if ((lane >> 3) == j) mine = x;
-    }
-    if (base + lane * 16 < total) codes[(base >> 4) + lane] = mine;
-
-    // Zero counts and scales, one writer per group.
-    if constexpr (G <= 128) {
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        int t = zc[j];
-#pragma unroll
-        for (int off = 1; off < G / 4; off <<= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
-        const int64_t e = base + j * 128 + lane * 4;
-        if ((lane & (G / 4 - 1)) == 0 && e < total) {
-          scales[e / G] = s[j];
-          zeros[e / G] = t;
+      for (int off = 1; off < kLanesPerGroup; off <<= 1) zc += __shfl_xor_sync(0xffffffffu, zc, off);
+      if (e < total) {
+        codes[e >> 4] = word;
+        if ((lane & (kLanesPerGroup - 1)) == 0) {
+          scales[e / G] = s;
+          zeros[e / G] = zc;
         }
-      }
-    } else if constexpr (G == 256) {
-      int t0 = zc[0] + zc[1], t1 = zc[2] + zc[3];
-#pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {
-        t0 += __shfl_xor_sync(0xffffffffu, t0, off);
-        t1 += __shfl_xor_sync(0xffffffffu, t1, off);
-      }
-      if (lane == 0) {
-        scales[base / G] = s[0];
-        zeros[base / G] = t0;
-        if (base + G < total) {
-          scales[base / G + 1] = s[2];
-          zeros[base / G + 1] = t1;
-        }
-      }
-    } else {
-      int t = (zc[0] + zc[1]) + (zc[2] + zc[3]);
-#pragma unroll
-      for (int off = 1; off < 32; off <<= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
-      if (lane == 0) {
-        scales[base / G] = s[0];
-        zeros[base / G] = t;
       }
     }
   }
@@ -148,8 +99,9 @@ template <int G>
 cudaError_t launch(const float* w, int64_t total, uint32_t* codes, float* scales, int32_t* zeros,
                    int num_sms, cudaStream_t stream) {
   const int64_t nunits = (total + kUnit - 1) / kUnit;
+  const int64_t warps_needed = (nunits + kUnroll - 1) / kUnroll;
   const int64_t warps_per_block = kThreads / 32;
-  int64_t blocks = (nunits + warps_per_block - 1) / warps_per_block;
+  int64_t blocks = (warps_needed + warps_per_block - 1) / warps_per_block;
   const int64_t cap = static_cast<int64_t>(num_sms) * 8;  // 8 resident blocks per SM
   if (blocks > cap) blocks = cap;
   quantize_kernel<G><<<static_cast<unsigned>(blocks), kThreads, 0, stream>>>(w, total, codes,

@@ -162,8 +162,8 @@ tq_status fwd_checked(const void* x, int64_t m, int64_t k, const uint32_t* codes
     return e == cudaSuccess ? TQ_OK : cuda_fail(e, "cudaMemsetAsync");
   }
   const int bn = tq::ts_tile_tokens(m);
-  if ((m + bn - 1) / bn > 65535) return fail(TQ_ERR_UNSUPPORTED, "m=%lld too large", (long long)m);
-  if ((n + 127) / 128 > 2147483647LL) return fail(TQ_ERR_UNSUPPORTED, "n too large");
+  if (((n + 127) / 128) * ((m + bn - 1) / bn) >= (int64_t(1) << 31))
+    return fail(TQ_ERR_UNSUPPORTED, "too many output tiles (m=%lld n=%lld)", (long long)m, (long long)n);
   CUtensorMap tb, tc;
   TQ_TRY(make_map(&tb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, x, k, m, 64, bn,
                   CU_TENSOR_MAP_SWIZZLE_128B));
@@ -179,7 +179,7 @@ tq_status fwd_checked(const void* x, int64_t m, int64_t k, const uint32_t* codes
   a.m = m;
   a.log2g = log2_group(g);
   a.out_bf16 = y_dtype == TQ_OUT_BF16;
-  cudaError_t e = tq::launch_ts_gemm(tq::kTsFwd, bn, tb, tc, a, stream);
+  cudaError_t e = tq::launch_ts_gemm(tq::kTsFwd, bn, tb, tc, a, dev->num_sms, stream);
   return e == cudaSuccess ? TQ_OK : cuda_fail(e, "forward launch");
 }
 
@@ -301,7 +301,8 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
       if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
     } else {
       const int bn = tq::ts_tile_tokens(m);
-      if ((m + bn - 1) / bn > 65535) return fail(TQ_ERR_UNSUPPORTED, "m too large");
+      if (((k + 127) / 128) * ((m + bn - 1) / bn) >= (int64_t(1) << 31))
+        return fail(TQ_ERR_UNSUPPORTED, "too many output tiles (m=%lld k=%lld)", (long long)m, (long long)k);
       CUtensorMap tb, tc;
       TQ_TRY(make_map(&tb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, dy, n, m, 64, bn,
                       CU_TENSOR_MAP_SWIZZLE_128B));
@@ -317,7 +318,7 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
       a.m = m;
       a.log2g = log2_group(g);
       a.out_bf16 = dx_dtype == TQ_OUT_BF16;
-      cudaError_t e = tq::launch_ts_gemm(tq::kTsDx, bn, tb, tc, a, st);
+      cudaError_t e = tq::launch_ts_gemm(tq::kTsDx, bn, tb, tc, a, dev->num_sms, st);
       if (e != cudaSuccess) return cuda_fail(e, "dX launch");
     }
   }
@@ -328,8 +329,9 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
         if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
       }
     } else {
-      if ((n + tq::kDwTileN - 1) / tq::kDwTileN > 65535)
-        return fail(TQ_ERR_UNSUPPORTED, "n too large");
+      if (((n + tq::kDwTileN - 1) / tq::kDwTileN) * ((k + tq::kDwTileK - 1) / tq::kDwTileK) >=
+          (int64_t(1) << 31))
+        return fail(TQ_ERR_UNSUPPORTED, "too many dW tiles (n=%lld k=%lld)", (long long)n, (long long)k);
       CUtensorMap tx, tdy;
       TQ_TRY(make_map(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, x, k, m, 64, 64,
                       CU_TENSOR_MAP_SWIZZLE_128B));
@@ -342,7 +344,7 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
       a.n = n;
       a.k = k;
       a.accumulate = accumulate_dw != 0;
-      cudaError_t e = tq::launch_dw_gemm(tx, tdy, a, st);
+      cudaError_t e = tq::launch_dw_gemm(tx, tdy, a, dev->num_sms, st);
       if (e != cudaSuccess) return cuda_fail(e, "dW launch");
     }
   }
