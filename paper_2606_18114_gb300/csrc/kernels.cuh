@@ -29,10 +29,10 @@ struct TsArgs {
 };
 
 // Tile of the activation operand along the token dimension.
-int ts_tile_tokens(int64_t m);
+int ts_tile_tokens(int mode, int64_t m);
 
 // tmap_b: bf16 activations [m][red] with box {64, bn}, 128-byte swizzle.
-// tmap_codes: uint32 codes [wn][wk/16] with box {4, 128} (fwd) or {8, 64} (dx).
+// tmap_codes: uint32 codes [wn][wk/16] with box {8, 128} (8 words x 128 rows).
 // Persistent: min(tiles, num_sms) CTAs.
 cudaError_t launch_ts_gemm(int mode, int bn, const CUtensorMap& tmap_b,
                            const CUtensorMap& tmap_codes, const TsArgs& args, int num_sms,

@@ -44,11 +44,29 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
                : "memory");
 }
 
+// The waiting thread is suspended (up to kSuspendHintNs, or until the phase
+// completes) instead of spinning, so waiting warps leave the issue slots to the
+// warps that work.
+constexpr uint32_t kSuspendHintNs = 1000000;  // 1 ms
+
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(kSuspendHintNs)
+      : "memory");
+  return ok != 0;
+}
+
+// Non-blocking probe of the phase.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}\n"
       : "=r"(ok)
       : "r"(bar), "r"(parity)
@@ -58,14 +76,35 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 
 // Wait until the phase of parity `parity` of `bar` has completed, or give up.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* status) {
-  if (mbar_try_wait(bar, parity)) return true;
+  if (mbar_test_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t n = 1; n < kWaitMaxPolls; ++n) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((n & 63u) == 0 && globaltimer_ns() - t0 > kWaitLimitNs) break;
+    if (globaltimer_ns() - t0 > kWaitLimitNs) break;
   }
   atomicExch(status, kStatusTimeout);
   return false;
+}
+
+// Warp-level wait: lane 0 waits (suspended) and the outcome is broadcast; the
+// __syncwarp orders lane 0's acquire before the other lanes' reads. One waiter
+// per warp instead of 32 keeps barrier traffic off the critical path.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, int* status) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, status) ? 1 : 0;
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  __syncwarp();
+  return ok != 0;
+}
+
+__device__ __forceinline__ bool warp_wait2(uint32_t bar0, uint32_t parity0, uint32_t bar1,
+                                           uint32_t parity1, int* status) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0)
+    ok = (mbar_wait(bar0, parity0, status) && mbar_wait(bar1, parity1, status)) ? 1 : 0;
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  __syncwarp();
+  return ok != 0;
 }
 
 // ------------------------------------------------------------------ TMA

@@ -161,13 +161,13 @@ tq_status fwd_checked(const void* x, int64_t m, int64_t k, const uint32_t* codes
     cudaError_t e = cudaMemsetAsync(y, 0, static_cast<size_t>(m) * n * ybytes, stream);
     return e == cudaSuccess ? TQ_OK : cuda_fail(e, "cudaMemsetAsync");
   }
-  const int bn = tq::ts_tile_tokens(m);
+  const int bn = tq::ts_tile_tokens(tq::kTsFwd, m);
   if (((n + 127) / 128) * ((m + bn - 1) / bn) >= (int64_t(1) << 31))
     return fail(TQ_ERR_UNSUPPORTED, "too many output tiles (m=%lld n=%lld)", (long long)m, (long long)n);
   CUtensorMap tb, tc;
   TQ_TRY(make_map(&tb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, x, k, m, 64, bn,
                   CU_TENSOR_MAP_SWIZZLE_128B));
-  TQ_TRY(make_map(&tc, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, codes, k / 16, n, 4, 128,
+  TQ_TRY(make_map(&tc, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, codes, k / 16, n, 8, 128,
                   CU_TENSOR_MAP_SWIZZLE_NONE));
   tq::TsArgs a = *proto;
   a.codes = codes;
@@ -300,13 +300,13 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
       cudaError_t e = cudaMemsetAsync(dx, 0, static_cast<size_t>(m) * k * dxb, st);
       if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
     } else {
-      const int bn = tq::ts_tile_tokens(m);
+      const int bn = tq::ts_tile_tokens(tq::kTsDx, m);
       if (((k + 127) / 128) * ((m + bn - 1) / bn) >= (int64_t(1) << 31))
         return fail(TQ_ERR_UNSUPPORTED, "too many output tiles (m=%lld k=%lld)", (long long)m, (long long)k);
       CUtensorMap tb, tc;
       TQ_TRY(make_map(&tb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, dy, n, m, 64, bn,
                       CU_TENSOR_MAP_SWIZZLE_128B));
-      TQ_TRY(make_map(&tc, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, codes, k / 16, n, 8, 64,
+      TQ_TRY(make_map(&tc, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, codes, k / 16, n, 8, 128,
                       CU_TENSOR_MAP_SWIZZLE_NONE));
       tq::TsArgs a{};
       a.codes = codes;

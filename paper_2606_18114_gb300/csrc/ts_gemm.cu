@@ -2,19 +2,19 @@
 // ternary weights expanded on chip straight into tensor memory.
 //
 // Output tile: 128 weight rows (TMEM lanes) x BN tokens (TMEM columns), fp32
-// accumulator D^T[row][token] in TMEM, two accumulators so that the epilogue of
-// one tile overlaps the main loop of the next. One CTA per SM walks the tiles
+// accumulator D^T[row][token] in TMEM. One CTA per SM walks the tiles
 // (rows fastest, so the CTAs in flight share the activation tile in L2). Per
-// 64-wide slice of the reduction ("k-block"):
-//   * warp 0 (one lane) TMA-loads the activation tile [BN tokens][64] (128-byte
-//     swizzle, K-major B operand) and the packed codes of the slice into one
-//     shared-memory stage;
-//   * warps 6-13, two warpgroups taking alternate k-blocks (warp w owns TMEM
-//     lanes 32*(w%4)..+31), expand the codes of their rows to bf16 pairs
-//     bf16(s)*c and tcgen05.st them into the stage's 32 TMEM columns (A operand,
-//     K-major, two bf16 per column);
-//   * warp 1 (one lane) issues four 128 x BN x 16 tcgen05.mma (A from TMEM, B
-//     from shared memory) and commits them to the stage's "empty" barrier;
+// 128-wide slice of the reduction ("k-block"):
+//   * warp 0 (one lane) TMA-loads the activation tile [BN tokens][128] (two
+//     64-wide boxes with the 128-byte swizzle, K-major B operand) and the packed
+//     codes of the slice into one shared-memory stage;
+//   * warps 6-13, two warpgroups each covering half of the slice (warp w owns
+//     TMEM lanes 32*(w%4)..+31), expand the codes of their rows to bf16 pairs
+//     bf16(s)*c as soon as the codes land, and tcgen05.st them into the A stage
+//     (K-major, two bf16 per column) once the MMAs that last read it are done;
+//   * warp 1 (one lane) issues eight 128 x BN x 16 tcgen05.mma (A from TMEM, B
+//     from shared memory) and one commit, which frees the smem stage and, later,
+//     the A stage;
 //   * warps 2-5 (one warpgroup) drain the finished accumulator with tcgen05.ld
 //     and store it; each warp store covers 32 consecutive rows of one token.
 // The expanded weights never touch shared memory, so shared-memory bandwidth is
@@ -41,25 +41,42 @@ namespace {
 constexpr int kEpiWarp0 = 2;                 // warps 2..5: epilogue warpgroup
 constexpr int kExpWarp0 = 6;                 // warps 6..13: two expansion warpgroups
 constexpr int kThreads = 14 * 32;
-constexpr int kStages = 4;
-constexpr int kKBlock = 64;                  // reduction elements per stage
-constexpr int kCodesBytes = 2048;            // 128 x 16 B (fwd) or 64 x 32 B (dx)
+constexpr int kKBlock = 128;                 // reduction elements per stage
+constexpr int kCodesBytes = 4096;            // 128 rows x 8 code words
 
-template <int BN>
+// Rings: kSmem shared-memory stages (activation tile as two 64-wide swizzled halves
+// + codes, filled by TMA) and kAStages tensor-memory stages of expanded weights
+// (64 columns = 128 k each). Each stage's MMAs are committed to the smem stage's
+// "empty" barrier (refill by TMA); when the smem ring is at least as deep as the
+// A ring, that same commit tells the expansion, kAStages iterations later, that
+// the A stage is free, otherwise a second commit goes to the A stage's barrier.
+// Tensor memory (512 columns) holds kAcc accumulators of BN columns plus the A ring:
+//   forward, 192 tokens: two accumulators (the epilogue, which writes the large
+//     fp32 Y, overlaps the next tile) and two A stages;
+//   dX, 256 tokens: one accumulator and four A stages (long tiles over the
+//     8512-wide reduction, so the serial epilogue is cheap and a deep A ring
+//     hides the commit -> expansion -> MMA round trip);
+//   decode, 16 tokens: two accumulators and four A stages.
+template <int MODE, int BN>
 struct TsLayout {
-  static constexpr int kBBytes = BN * kKBlock * 2;
+  static constexpr int kSmem = BN == 16 ? 16 : (BN == 192 ? 4 : 3);
+  static constexpr int kAStages = BN == 192 ? 2 : 4;
+  static constexpr int kAcc = BN == 256 ? 1 : 2;
+  static constexpr bool kReleaseViaSmem = kSmem >= kAStages;
+  static constexpr int kSubBytes = BN * 64 * 2;                // one 64-wide k half
+  static constexpr int kBBytes = 2 * kSubBytes;
   static constexpr int kStageBytes = ((kBBytes + kCodesBytes + 1023) / 1024) * 1024;
-  static constexpr int kScaleOff = kStages * kStageBytes;   // dx: 2 WG x 4 warps x 2 x 64 bf16
+  static constexpr int kScaleOff = kSmem * kStageBytes;     // dx: 2 WG x 4 warps x 2 x 64 bf16
   static constexpr int kScaleBytes = 2 * 4 * 2 * 64 * 2;
   static constexpr int kBarOff = kScaleOff + kScaleBytes;
-  static constexpr int kNumBars = 3 * kStages + 4;
+  static constexpr int kNumBars = 2 * kSmem + 2 * kAStages + 2 * kAcc;
   static constexpr int kBytes = kBarOff + kNumBars * 8 + 8;
   static constexpr int kTxBytes = kBBytes + kCodesBytes;
-  static constexpr int kTmemNeed = 2 * BN + kStages * 32;
+  static constexpr int kTmemNeed = kAcc * BN + kAStages * 64;
   static constexpr uint32_t kTmemCols = kTmemNeed <= 32 ? 32 : kTmemNeed <= 64 ? 64
                                         : kTmemNeed <= 128 ? 128 : kTmemNeed <= 256 ? 256 : 512;
   static_assert(kTmemNeed <= 512, "tensor memory");
-  static_assert(BN % 32 == 0 || BN == 16, "epilogue chunks");
+  static_assert(BN % 16 == 0, "epilogue chunks");
 };
 
 __device__ __forceinline__ uint32_t bmul2(uint32_t a, uint32_t b) {
@@ -82,18 +99,12 @@ __device__ __forceinline__ void expand_word(uint32_t w, uint32_t hs, uint32_t* a
   for (int j = 0; j < 8; ++j) a[j] = bmul2((w << (14 - 2 * j)) & 0xC000C000u, hs);
 }
 
-__device__ __forceinline__ void store_out(void* out, int64_t idx, float v, int bf16) {
-  if (bf16)
-    static_cast<__nv_bfloat16*>(out)[idx] = __float2bfloat16_rn(v);
-  else
-    static_cast<float*>(out)[idx] = v;
-}
-
 template <int MODE, int BN>
 __global__ void __launch_bounds__(kThreads, 1)
     ts_gemm_kernel(const __grid_constant__ CUtensorMap tmap_b,
                    const __grid_constant__ CUtensorMap tmap_codes, const TsArgs args) {
-  using L = TsLayout<BN>;
+  using L = TsLayout<MODE, BN>;
+  constexpr int kSmem = L::kSmem, kAS = L::kAStages, kAcc = L::kAcc;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -106,7 +117,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   // tokens (t / row_tiles) * BN; tile counts fit in 32 bits (checked on the host)
   const uint32_t row_tiles = static_cast<uint32_t>((rows + 127) / 128);
   const uint32_t tiles = row_tiles * static_cast<uint32_t>((args.m + BN - 1) / BN);
-  const int my_tiles = blockIdx.x < tiles ? static_cast<int>((tiles - 1 - blockIdx.x) / gridDim.x + 1) : 0;
+  const int my_tiles =
+      blockIdx.x < tiles ? static_cast<int>((tiles - 1 - blockIdx.x) / gridDim.x + 1) : 0;
   const int total = my_tiles * nkb;  // k-blocks this CTA runs
   int* status = args.status;
   auto tile_r0 = [&](int i) -> int64_t {
@@ -119,21 +131,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t smem_base = smem_u32(smem);
   const uint32_t bar_base = smem_base + L::kBarOff;
   auto full_bar = [&](int s) { return bar_base + 8u * s; };
-  auto empty_bar = [&](int s) { return bar_base + 8u * (kStages + s); };
-  auto afull_bar = [&](int s) { return bar_base + 8u * (2 * kStages + s); };
-  auto accfull_bar = [&](int a) { return bar_base + 8u * (3 * kStages + a); };
-  auto accempty_bar = [&](int a) { return bar_base + 8u * (3 * kStages + 2 + a); };
+  auto empty_bar = [&](int s) { return bar_base + 8u * (kSmem + s); };
+  auto afull_bar = [&](int a) { return bar_base + 8u * (2 * kSmem + a); };
+  auto aempty_bar = [&](int a) { return bar_base + 8u * (2 * kSmem + kAS + a); };
+  auto accfull_bar = [&](int a) { return bar_base + 8u * (2 * kSmem + 2 * kAS + a); };
+  auto accempty_bar = [&](int a) { return bar_base + 8u * (2 * kSmem + 2 * kAS + kAcc + a); };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::kBarOff + L::kNumBars * 8);
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < kSmem; ++s) {
       mbar_init(full_bar(s), 1);
       mbar_init(empty_bar(s), 1);
-      mbar_init(afull_bar(s), 128);
     }
-    for (int a = 0; a < 2; ++a) {
+    for (int a = 0; a < kAS; ++a) {
+      mbar_init(afull_bar(a), 8);  // one arrival per expansion warp
+      mbar_init(aempty_bar(a), 1);
+    }
+    for (int a = 0; a < kAcc; ++a) {
       mbar_init(accfull_bar(a), 1);
-      mbar_init(accempty_bar(a), 128);
+      mbar_init(accempty_bar(a), 4);  // one arrival per epilogue warp
     }
     fence_mbar_init();
   }
@@ -149,7 +165,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const uint32_t tmem_a = tmem_base + 2 * BN;
+  const uint32_t tmem_a = tmem_base + kAcc * BN;
 
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer
@@ -158,13 +174,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int it = 0; it < total; ++it) {
         const int i = it / nkb, kb = it - i * nkb;
-        const int s = it % kStages;
-        const uint32_t ph = (it / kStages) & 1;
+        const int s = it % kSmem;
+        const uint32_t ph = (it / kSmem) & 1;
         if (!(ok = mbar_wait(empty_bar(s), ph ^ 1, status))) break;
         const uint32_t stage = smem_base + s * L::kStageBytes;
         const int64_t r0 = tile_r0(i), m0 = tile_m0(i);
         mbar_arrive_expect_tx(full_bar(s), L::kTxBytes);
         tma_load_2d(stage, &tmap_b, full_bar(s), kb * kKBlock, static_cast<int32_t>(m0));
+        tma_load_2d(stage + L::kSubBytes, &tmap_b, full_bar(s), kb * kKBlock + 64,
+                    static_cast<int32_t>(m0));
         if (MODE == kTsFwd)
           tma_load_2d(stage + L::kBBytes, &tmap_codes, full_bar(s), kb * (kKBlock / 16),
                       static_cast<int32_t>(r0));
@@ -174,8 +192,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++issued;
       }
       if (!ok) {  // let copies already in flight land before the CTA winds down
-        for (int it = issued - 1; it >= 0 && it >= issued - kStages; --it)
-          mbar_wait(full_bar(it % kStages), (it / kStages) & 1, status);
+        for (int it = issued - 1; it >= 0 && it >= issued - kSmem; --it)
+          mbar_wait(full_bar(it % kSmem), (it / kSmem) & 1, status);
       }
     }
   } else if (warp == 1) {
@@ -185,24 +203,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       int it = 0;
       bool ok = true;
       for (int i = 0; i < my_tiles && ok; ++i) {
-        const int acc = i & 1;
-        const uint32_t aph = (i >> 1) & 1;
+        const int acc = i % kAcc;
+        const uint32_t aph = (i / kAcc) & 1;
         if (!(ok = mbar_wait(accempty_bar(acc), aph ^ 1, status))) break;
         tc_fence_after();
         const uint32_t d = tmem_base + acc * BN;
         for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const int s = it % kStages;
-          const uint32_t ph = (it / kStages) & 1;
-          if (!(ok = mbar_wait(full_bar(s), ph, status) && mbar_wait(afull_bar(s), ph, status)))
-            break;
+          const int s = it % kSmem, as = it % kAS;
+          // afull implies full: the expansion warps waited on this stage's TMA
+          // barrier before they arrived, so one wait orders both operands.
+          if (!(ok = mbar_wait(afull_bar(as), (it / kAS) & 1, status))) break;
           tc_fence_after();
           const uint32_t b_addr = smem_base + s * L::kStageBytes;
 #pragma unroll
           for (int j = 0; j < kKBlock / 16; ++j) {
-            const uint64_t bdesc = smem_desc_sw128(b_addr + j * 32, 16, 1024);
-            mma_ts(d, tmem_a + s * 32 + j * 8, bdesc, idesc, (kb | j) != 0);
+            const uint64_t bdesc =
+                smem_desc_sw128(b_addr + (j >> 2) * L::kSubBytes + (j & 3) * 32, 16, 1024);
+            mma_ts(d, tmem_a + as * 64 + j * 8, bdesc, idesc, (kb | j) != 0);
           }
           mma_commit(empty_bar(s));
+          if (!L::kReleaseViaSmem) mma_commit(aempty_bar(as));
         }
         if (ok) mma_commit(accfull_bar(acc));
       }
@@ -213,96 +233,131 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     const int64_t m = args.m;
     for (int i = 0; i < my_tiles; ++i) {
-      const int acc = i & 1;
-      const uint32_t aph = (i >> 1) & 1;
-      if (!__all_sync(0xffffffffu, mbar_wait(accfull_bar(acc), aph, status))) break;
+      const int acc = i % kAcc;
+      const uint32_t aph = (i / kAcc) & 1;
+      if (!warp_wait(accfull_bar(acc), aph, status)) break;
       tc_fence_after();
       const int64_t row = tile_r0(i) + quad * 32 + lane;
       const int64_t m0 = tile_m0(i);
       const uint32_t d = tmem_base + acc * BN + lane_off;
-      if (BN == 16) {
-        uint32_t v[32] = {};
-        tmem_ld_x16(d, v);
-        tmem_ld_wait(v);
-        if (row < rows) {
-#pragma unroll
-          for (int t = 0; t < 16; ++t)
-            if (m0 + t < m)
-              store_out(args.out, (m0 + t) * rows + row, __uint_as_float(v[t]), args.out_bf16);
-        }
-      } else {
+      // element (m0 + c + t, row) of out; tokens beyond m are not stored
+      const int mvalid = static_cast<int>(m - m0 < BN ? m - m0 : BN);
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 16) {
-          uint32_t v[16];
-          tmem_ld16(d + c, v);
-          tmem_ld_wait16(v);
-          if (row < rows) {
+      for (int c = 0; c < BN; c += 16) {
+        uint32_t v[16];
+        tmem_ld16(d + c, v);
+        tmem_ld_wait16(v);
+        if (row < rows) {
+          if (args.out_bf16) {
+            __nv_bfloat16* p = static_cast<__nv_bfloat16*>(args.out) + (m0 + c) * rows + row;
 #pragma unroll
-            for (int t = 0; t < 16; ++t)
-              if (m0 + c + t < m)
-                store_out(args.out, (m0 + c + t) * rows + row, __uint_as_float(v[t]),
-                          args.out_bf16);
+            for (int t = 0; t < 16; ++t, p += rows)
+              if (c + t < mvalid) *p = __float2bfloat16_rn(__uint_as_float(v[t]));
+          } else {
+            float* p = static_cast<float*>(args.out) + (m0 + c) * rows + row;
+#pragma unroll
+            for (int t = 0; t < 16; ++t, p += rows)
+              if (c + t < mvalid) *p = __uint_as_float(v[t]);
           }
         }
       }
       tc_fence_before();
-      mbar_arrive(accempty_bar(acc));
+      __syncwarp();
+      if (lane == 0) mbar_arrive(accempty_bar(acc));
     }
   } else {
     // ---------------------------------------------------------------- expansion
-    const int wg = (warp - kExpWarp0) >> 2;   // 0 or 1: takes k-blocks it % 2 == wg
+    // Both warpgroups take every k-block: warpgroup wg fills A columns
+    // [32 wg, 32 wg + 32) of the stage, i.e. reduction offsets [64 wg, 64 wg + 64).
+    const int wg = (warp - kExpWarp0) >> 2;
     const int quad = warp & 3;
     const int r_local = quad * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     const int64_t gpr = args.wk >> args.log2g;  // groups per weight row
 
+    // Cursor over k-blocks: tile i, k-block kb, first row of the tile.
+    struct Cursor {
+      int it, i, kb;
+      int64_t r0;
+    };
+    auto cursor_at = [&](int it) {
+      Cursor c;
+      c.it = it;
+      c.i = it / nkb;
+      c.kb = it - c.i * nkb;
+      c.r0 = tile_r0(c.i);
+      return c;
+    };
+    auto advance = [&](Cursor& c) {
+      ++c.it;
+      if (++c.kb == nkb) {
+        c.kb = 0;
+        ++c.i;
+        c.r0 = tile_r0(c.i);
+      }
+    };
+    // The A stage of iteration it is free once the MMAs of iteration it - kAS are done.
+    auto a_free = [&](int it) -> bool {
+      if (L::kReleaseViaSmem) {
+        if (it < kAS) return true;
+        const int j = it - kAS;
+        return warp_wait(empty_bar(j % kSmem), (j / kSmem) & 1, status);
+      }
+      return warp_wait(aempty_bar(it % kAS), ((it / kAS) & 1) ^ 1, status);
+    };
+    auto publish = [&](int as, const uint32_t* a) {
+      tc_fence_after();
+      tmem_st_x16(tmem_a + as * 64 + wg * 32 + lane_off, a);
+      tmem_st_x16(tmem_a + as * 64 + wg * 32 + 16 + lane_off, a + 16);
+      tmem_st_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(afull_bar(as));
+    };
+    Cursor cur = cursor_at(0);
+    Cursor pre = cursor_at(2);
+
     if (MODE == kTsFwd) {
-      auto load_sc = [&](int it) -> float2 {
-        if (it >= total) return make_float2(0.f, 0.f);
-        const int i = it / nkb, kb = it - i * nkb;
-        const int64_t row = tile_r0(i) + r_local;
-        if (row >= args.wn) return make_float2(0.f, 0.f);
+      auto load_sc = [&](const Cursor& c) -> float2 {
+        const int64_t row = c.r0 + r_local;
+        if (c.it >= total || row >= args.wn) return make_float2(0.f, 0.f);
         const float* srow = args.scales + row * gpr;
-        const int64_t gi = (static_cast<int64_t>(kb) * kKBlock) >> args.log2g;
+        const int64_t gi = (static_cast<int64_t>(c.kb) * kKBlock + wg * 64) >> args.log2g;
         if (args.log2g == 5) return __ldg(reinterpret_cast<const float2*>(srow + gi));
         const float x = __ldg(srow + gi);
         return make_float2(x, x);
       };
-      float2 p0 = load_sc(wg), p1 = load_sc(wg + 2);
-      for (int it = wg; it < total; it += 2) {
-        const int s = it % kStages;
-        const uint32_t ph = (it / kStages) & 1;
+      float2 p0 = load_sc(cur), p1 = load_sc(cursor_at(1));
+      for (; cur.it < total; advance(cur), advance(pre)) {
+        const int it = cur.it;
+        const int s = it % kSmem, as = it % kAS;
         const float2 sc = p0;
         p0 = p1;
-        p1 = load_sc(it + 4);
-        const bool got = mbar_wait(empty_bar(s), ph ^ 1, status) && mbar_wait(full_bar(s), ph, status);
-        if (!__all_sync(0xffffffffu, got)) break;
-        tc_fence_after();
+        p1 = load_sc(pre);
+        // Expand as soon as the codes have landed; only the tensor-memory store
+        // waits for the A stage.
+        if (!warp_wait(full_bar(s), (it / kSmem) & 1, status)) break;
         const uint4 cw = *reinterpret_cast<const uint4*>(smem + s * L::kStageBytes + L::kBBytes +
-                                                         r_local * 16);
+                                                         r_local * 32 + wg * 16);
         const uint32_t hs_lo = half_scale_pair(sc.x, sc.x);
         const uint32_t hs_hi = half_scale_pair(sc.y, sc.y);
-        uint32_t a[16];
+        uint32_t a[32];
         expand_word(cw.x, hs_lo, a + 0);
         expand_word(cw.y, hs_lo, a + 8);
-        tmem_st_x16(tmem_a + s * 32 + lane_off, a);
-        expand_word(cw.z, hs_hi, a + 0);
-        expand_word(cw.w, hs_hi, a + 8);
-        tmem_st_x16(tmem_a + s * 32 + 16 + lane_off, a);
-        tmem_st_wait();
-        tc_fence_before();
-        mbar_arrive(afull_bar(s));
+        expand_word(cw.z, hs_hi, a + 16);
+        expand_word(cw.w, hs_hi, a + 24);
+        if (!a_free(it)) break;
+        publish(as, a);
       }
     } else {
-      // dX: this thread is input feature k = row; a warp shares one k-group.
-      auto load_sc = [&](int it) -> float2 {
+      // dX: this thread is input feature k = row; a warp shares one k-group, and
+      // warpgroup wg covers rows n in [kb*128 + 64 wg, kb*128 + 64 wg + 64).
+      auto load_sc = [&](const Cursor& c) -> float2 {
         float2 r = make_float2(0.f, 0.f);
-        if (it >= total) return r;
-        const int i = it / nkb, kb = it - i * nkb;
-        const int64_t kwarp = tile_r0(i) + quad * 32;
-        if (kwarp >= args.wk) return r;
+        const int64_t kwarp = c.r0 + quad * 32;
+        if (c.it >= total || kwarp >= args.wk) return r;
         const int64_t gk = kwarp >> args.log2g;
-        const int64_t n_a = static_cast<int64_t>(kb) * kKBlock + lane;
+        const int64_t n_a = static_cast<int64_t>(c.kb) * kKBlock + wg * 64 + lane;
         const int64_t n_b = n_a + 32;
         if (n_a < args.wn) r.x = __ldg(args.scales + n_a * gpr + gk);
         if (n_b < args.wn) r.y = __ldg(args.scales + n_b * gpr + gk);
@@ -316,40 +371,31 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int xw = r_local >> 4;
       __nv_bfloat16* sbuf =
           reinterpret_cast<__nv_bfloat16*>(smem + L::kScaleOff) + (wg * 4 + quad) * 128;
-      float2 p0 = load_sc(wg), p1 = load_sc(wg + 2);
-      int local = 0;
-      for (int it = wg; it < total; it += 2, ++local) {
-        const int s = it % kStages;
-        const uint32_t ph = (it / kStages) & 1;
+      float2 p0 = load_sc(cur), p1 = load_sc(cursor_at(1));
+      for (; cur.it < total; advance(cur), advance(pre)) {
+        const int it = cur.it;
+        const int s = it % kSmem, as = it % kAS;
         const float2 sc = p0;
         p0 = p1;
-        p1 = load_sc(it + 4);
-        __nv_bfloat16* sb = sbuf + (local & 1) * 64;
+        p1 = load_sc(pre);
+        __nv_bfloat16* sb = sbuf + (it & 1) * 64;
         sb[lane] = __float2bfloat16_rn(0.5f * sc.x);
         sb[lane + 32] = __float2bfloat16_rn(0.5f * sc.y);
         __syncwarp();
-        const bool got = mbar_wait(empty_bar(s), ph ^ 1, status) && mbar_wait(full_bar(s), ph, status);
-        if (!__all_sync(0xffffffffu, got)) break;
-        tc_fence_after();
+        if (!warp_wait(full_bar(s), (it / kSmem) & 1, status)) break;
         const uint32_t* tile =
-            reinterpret_cast<const uint32_t*>(smem + s * L::kStageBytes + L::kBBytes);
+            reinterpret_cast<const uint32_t*>(smem + s * L::kStageBytes + L::kBBytes) + wg * 64 * 8;
         const uint32_t* spair = reinterpret_cast<const uint32_t*>(sb);
+        uint32_t a[32];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          uint32_t a[16];
-#pragma unroll
-          for (int q = 0; q < 16; ++q) {
-            const int p = 16 * h + q;
-            const uint32_t w0 = tile[(2 * p) * 8 + xw];
-            const uint32_t w1 = tile[(2 * p + 1) * 8 + xw];
-            const uint32_t t = (__byte_perm(w0, w1, sel) << shift) & 0xC000C000u;
-            a[q] = bmul2(t, spair[p]);
-          }
-          tmem_st_x16(tmem_a + s * 32 + 16 * h + lane_off, a);
+        for (int p = 0; p < 32; ++p) {
+          const uint32_t w0 = tile[(2 * p) * 8 + xw];
+          const uint32_t w1 = tile[(2 * p + 1) * 8 + xw];
+          const uint32_t t = (__byte_perm(w0, w1, sel) << shift) & 0xC000C000u;
+          a[p] = bmul2(t, spair[p]);
         }
-        tmem_st_wait();
-        tc_fence_before();
-        mbar_arrive(afull_bar(s));
+        if (!a_free(it)) break;
+        publish(as, a);
       }
     }
   }
@@ -366,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 template <int MODE, int BN>
 cudaError_t launch_impl(const CUtensorMap& tb, const CUtensorMap& tc, const TsArgs& a,
                         int num_sms, cudaStream_t stream) {
-  using L = TsLayout<BN>;
+  using L = TsLayout<MODE, BN>;
   // Enough shared memory that two CTAs never share an SM (each holds up to 512
   // tensor-memory columns).
   size_t smem = L::kBytes + 1024;
@@ -384,7 +430,7 @@ cudaError_t launch_impl(const CUtensorMap& tb, const CUtensorMap& tc, const TsAr
 
 }  // namespace
 
-int ts_tile_tokens(int64_t m) { return m <= 16 ? 16 : 192; }
+int ts_tile_tokens(int mode, int64_t m) { return m <= 16 ? 16 : (mode == kTsFwd ? 192 : 256); }
 
 cudaError_t launch_ts_gemm(int mode, int bn, const CUtensorMap& tb, const CUtensorMap& tc,
                            const TsArgs& a, int num_sms, cudaStream_t stream) {
@@ -393,7 +439,7 @@ cudaError_t launch_ts_gemm(int mode, int bn, const CUtensorMap& tb, const CUtens
     if (bn == 192) return launch_impl<kTsFwd, 192>(tb, tc, a, num_sms, stream);
   } else {
     if (bn == 16) return launch_impl<kTsDx, 16>(tb, tc, a, num_sms, stream);
-    if (bn == 192) return launch_impl<kTsDx, 192>(tb, tc, a, num_sms, stream);
+    if (bn == 256) return launch_impl<kTsDx, 256>(tb, tc, a, num_sms, stream);
   }
   return cudaErrorInvalidValue;
 }
