@@ -38,6 +38,32 @@ cudaError_t launch_ts_gemm(int mode, int bn, const CUtensorMap& tmap_b,
                            const CUtensorMap& tmap_codes, const TsArgs& args, int num_sms,
                            cudaStream_t stream);
 
+// decode.cu ------------------------------------------------------------------
+// Forward for m <= 16 tokens over one or many matrices in one launch.
+struct DecodeMat {
+  const uint32_t* codes;  // uint32 [n][k/16]
+  const float* scales;    // fp32 [n][k/g]
+  const void* x;          // bf16 [m][k]
+  void* y;                // [m][n], fp32 or bf16
+  int64_t n, k;           // k % 64 == 0
+  int32_t log2g;
+  int32_t y_bf16;
+  int32_t unit0;          // first 16-row unit of this matrix in the batch
+  int32_t pad;
+};
+
+constexpr int kDecodeMaxMats = 256;
+
+struct DecodeBatch {
+  DecodeMat mats[kDecodeMaxMats];
+  int32_t count;
+  int32_t m;              // tokens, 1..16
+  int32_t total_units;    // sum over matrices of ceil(n / 16)
+  int32_t pad;
+};
+
+cudaError_t launch_decode(const DecodeBatch& batch, int num_sms, cudaStream_t stream);
+
 // dw_gemm.cu -----------------------------------------------------------------
 // dW[n][k] (+)= sum_m dy[m][n] x[m][k], both operands MN-major from TMA.
 struct DwArgs {

@@ -183,6 +183,46 @@ tq_status fwd_checked(const void* x, int64_t m, int64_t k, const uint32_t* codes
   return e == cudaSuccess ? TQ_OK : cuda_fail(e, "forward launch");
 }
 
+static_assert(tq::kDecodeMaxMats >= TQ_MAX_BATCH, "decode batch table");
+
+// Forward for m <= 16 tokens: the HBM-streaming decode kernel over all matrices.
+tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
+                         cudaStream_t stream) {
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  thread_local tq::DecodeBatch b;
+  int64_t units = 0;
+  int used = 0;
+  for (int32_t i = 0; i < count; ++i) {
+    const tq_fwd_desc& d = descs[i];
+    if (d.n == 0) continue;
+    if (d.k == 0) {
+      const size_t yb = d.y_dtype == TQ_OUT_BF16 ? 2 : 4;
+      cudaError_t e = cudaMemsetAsync(d.y, 0, static_cast<size_t>(m) * d.n * yb, stream);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+      continue;
+    }
+    tq::DecodeMat& dm = b.mats[used++];
+    dm.codes = d.codes;
+    dm.scales = d.scales;
+    dm.x = d.x;
+    dm.y = d.y;
+    dm.n = d.n;
+    dm.k = d.k;
+    dm.log2g = log2_group(d.g);
+    dm.y_bf16 = d.y_dtype == TQ_OUT_BF16;
+    dm.unit0 = static_cast<int32_t>(units);
+    units += (d.n + 15) / 16;
+    if (units >= (int64_t(1) << 31)) return fail(TQ_ERR_UNSUPPORTED, "too many decode rows");
+  }
+  if (used == 0) return TQ_OK;
+  b.count = used;
+  b.m = static_cast<int32_t>(m);
+  b.total_units = static_cast<int32_t>(units);
+  cudaError_t e = tq::launch_decode(b, dev->num_sms, stream);
+  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "decode launch");
+}
+
 tq_status check_fwd_args(const void* x, int64_t m, int64_t k, const uint32_t* codes,
                          const float* scales, int64_t n, int32_t g, const void* y,
                          int32_t y_dtype) {
@@ -231,6 +271,10 @@ TQ_API tq_status tq_linear_fwd(const void* x, int64_t m, int64_t k, const uint32
                                int32_t y_dtype, void* stream) {
   g_err[0] = 0;
   TQ_TRY(check_fwd_args(x, m, k, codes, scales, n, g, y, y_dtype));
+  if (m >= 1 && m <= 16 && n > 0) {
+    tq_fwd_desc d{x, codes, scales, y, n, k, g, y_dtype};
+    return decode_checked(&d, 1, m, static_cast<cudaStream_t>(stream));
+  }
   tq::TsArgs proto{};
   return fwd_checked(x, m, k, codes, scales, n, g, y, y_dtype, static_cast<cudaStream_t>(stream),
                      &proto);
@@ -253,13 +297,7 @@ TQ_API tq_status tq_linear_fwd_batched(const tq_fwd_desc* descs, int32_t count, 
       return fail(st, "%s", msg);
     }
   }
-  tq::TsArgs proto{};
-  for (int32_t i = 0; i < count; ++i) {
-    const tq_fwd_desc& d = descs[i];
-    TQ_TRY(fwd_checked(d.x, m, d.k, d.codes, d.scales, d.n, d.g, d.y, d.y_dtype,
-                       static_cast<cudaStream_t>(stream), &proto));
-  }
-  return TQ_OK;
+  return decode_checked(descs, count, m, static_cast<cudaStream_t>(stream));
 }
 
 TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t n, int64_t k,

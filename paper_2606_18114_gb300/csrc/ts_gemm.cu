@@ -435,7 +435,6 @@ int ts_tile_tokens(int mode, int64_t m) { return m <= 16 ? 16 : (mode == kTsFwd 
 cudaError_t launch_ts_gemm(int mode, int bn, const CUtensorMap& tb, const CUtensorMap& tc,
                            const TsArgs& a, int num_sms, cudaStream_t stream) {
   if (mode == kTsFwd) {
-    if (bn == 16) return launch_impl<kTsFwd, 16>(tb, tc, a, num_sms, stream);
     if (bn == 192) return launch_impl<kTsFwd, 192>(tb, tc, a, num_sms, stream);
   } else {
     if (bn == 16) return launch_impl<kTsDx, 16>(tb, tc, a, num_sms, stream);

@@ -181,6 +181,40 @@ def test_empty_sizes(tq):
     assert float(dw.abs().max()) == 0.0   # M = 0: dW = empty sum = 0
 
 
+@pytest.mark.parametrize("g", [32, 64, 128, 256, 512])
+@pytest.mark.parametrize("m", [1, 5, 8, 9, 16])
+def test_decode_parity(tq, g, m):
+    """Few-token forward (decode kernel): ragged rows (200 = 12.5 units of 16)."""
+    n, k = 200, 1024
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=g + m)
+    y = tq.linear_fwd(x.cuda(), codes, s, g)
+    yb = tq.linear_fwd(x.cuda(), codes, s, g, out_dtype=torch.bfloat16)
+    tq.device_status()
+    ref = O.linear_fwd(x, w_hat)
+    check_close(y, ref, "Y decode")
+    assert torch.equal(yb, y.to(torch.bfloat16))
+
+
+def test_batched_decode_mixed(tq):
+    """One launch over matrices with different shapes, group sizes and output types."""
+    specs = [(520, 256, 128, torch.float32), (264, 512, 32, torch.bfloat16),
+             (8, 64, 64, torch.float32), (136, 1024, 512, torch.float32)]
+    items = []
+    for i, (n, k, g, dt) in enumerate(specs):
+        w = synth.latent_weights(n, k, seed=200 + i)
+        x = synth.activations_bf16(11, k, seed=200 + i)
+        codes, s, _ = _quant(tq, w, g)
+        ref = O.quantize(w, g)
+        items.append(dict(x=x.cuda(), codes=codes, scales=s, g=g,
+                          y=torch.empty((11, n), device="cuda", dtype=dt),
+                          ref=O.linear_fwd(x, O.dequantize(ref[0], ref[1], k, g))))
+    tq.linear_fwd_batched(items, 11)
+    tq.device_status()
+    for i, it in enumerate(items):
+        check_close(it["y"].float(), it["ref"], f"batched Y[{i}]",
+                    max_rel_rms=3e-2 if it["y"].dtype == torch.bfloat16 else 2e-2)
+
+
 def test_batched_decode_matches_single(tq):
     mats = []
     for i, (n, k) in enumerate([(520, 256), (256, 512), (520, 256), (136, 1024)]):
