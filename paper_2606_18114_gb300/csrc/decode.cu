@@ -3,24 +3,30 @@
 // the layer is bound by weight traffic; 2-bit codes + fp32 group scales are 0.28
 // bytes per weight at g = 128).
 //
-// Work unit = 16 consecutive weight rows of one matrix over its whole K; each warp
-// walks units u = global_warp, global_warp + warps, ... across all matrices.
-// Per 64-wide chunk of K a warp runs four mma.sync.m16n8k16 (bf16 in, fp32
-// accumulate) with the expanded weights as the 16 x 16 A operand and up to 8
-// tokens as the n8 B operand (two B tiles for 9..16 tokens).
+// Work unit = 16 consecutive weight rows of one matrix over its whole K. Each CTA
+// owns a contiguous range of units, balanced by their number of 128-wide chunks
+// of K (host-computed), so an SM works through one or two matrices at a time and
+// their x stays in L1. Warps take units from the range with a shared-memory
+// counter. A warp streams its units as a flat sequence of chunks: the codes of a
+// chunk (16 rows x 32 bytes) are one 16-byte cp.async per lane, zero-filled past
+// the matrix, into a per-warp ring of kDepth chunks (~128 KB per SM in flight
+// without holding registers); a per-warp queue hands the units claimed by the
+// prefetch cursor to the consuming cursor.
 //
+// Per chunk a warp runs eight mma.sync.m16n8k16 (bf16 in, fp32 accumulate) with
+// the expanded weights as the 16 x 16 A operand and up to 8 tokens as the n8 B
+// operand (two B tiles for 9..16 tokens), in two independent accumulator chains.
 // The reduction index of the MMA is permuted identically on both operands so that
-// lane (g, t) (g = lane / 4, t = lane % 4) consumes exactly code word t of the
-// chunk for rows g and g + 8 — reduction offsets 16t .. 16t + 15 — and the
-// contiguous 32 bytes x[token g][16t .. 16t + 15]: MMA number kb of the chunk
-// uses offsets 16t + 4kb + {0,1} for fragment slots (2t, 2t+1) and 16t + 4kb +
-// {2,3} for slots (2t+8, 2t+9). Code words and x are then read with coalesced
-// loads and no lane reads what another lane reads.
+// lane (g, t) (g = lane / 4, t = lane % 4) consumes exactly code words 2t, 2t+1 of
+// the chunk for rows g and g + 8 — reduction offsets 32t .. 32t + 31 — and the
+// contiguous 64 bytes x[token g][32t .. 32t + 31]: MMA kb takes offsets
+// 32t + 4kb + {0,1} for fragment slots (2t, 2t+1) and 32t + 4kb + {2,3} for slots
+// (2t+8, 2t+9).
 //
 // Expansion: pair j of a code word -> bf16x2 (2c, 2c) by ((w << (14 - 2j)) &
-// 0xC000C000) (layout of include/tq.h). For g >= 64 every chunk lies in one group,
-// so partial sums of a group are scaled by s/2 in fp32 (exact scale); for g = 32 the
-// two groups of a chunk meet inside one MMA, so the expansion multiplies by
+// 0xC000C000) (layout of include/tq.h). For g >= 128 a chunk lies in one group and
+// the partial sums of a group are scaled by s/2 in fp32 (exact scale); for g <= 64
+// the groups of a chunk meet inside one MMA, so the expansion multiplies by
 // bf16(s)/2 as the prefill kernels do.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -31,8 +37,12 @@
 namespace tq {
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kPrefetch = 6;   // chunks of code words in flight per warp
+constexpr int kWarps = 16;
+constexpr int kThreads = kWarps * 32;
+constexpr int kDepth = 16;                 // chunks in flight per warp
+constexpr int kChunkBytes = 16 * 32;       // 16 rows x 8 code words
+constexpr int kQueue = kDepth + 1;         // units claimed ahead of the consumer
+constexpr int kSmemBytes = kWarps * kDepth * kChunkBytes;
 
 __device__ __forceinline__ uint32_t bmul2(uint32_t a, uint32_t b) {
   uint32_t d;
@@ -40,23 +50,44 @@ __device__ __forceinline__ uint32_t bmul2(uint32_t a, uint32_t b) {
   return d;
 }
 
-__device__ __forceinline__ uint32_t pair_bits(uint32_t w, int j) {
-  return (w << (14 - 2 * j)) & 0xC000C000u;
+// Pair j of a code word as a bf16x2 of (2c, 2c): the mask keeps the pair's two
+// fields, the multiplication by mul = 2^(14 - 2j) moves them to bits 14-15 and
+// 30-31 (exact, the fields are 16 bits apart). mul is a register whose value the
+// compiler does not see, so the move runs as an integer multiply on the FMA pipe
+// instead of a shift on the ALU pipe, which the mask already loads.
+__device__ __forceinline__ uint32_t pair_bits(uint32_t w, int j, uint32_t mul) {
+  return (w & (0x00030003u << (2 * j))) * mul;
 }
 
-__device__ __forceinline__ void mma16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
-                                         uint32_t b1) {
+__device__ __forceinline__ uint32_t opaque(uint32_t v) {
+  uint32_t r;
+  asm volatile("mov.b32 %0, %1;" : "=r"(r) : "r"(v));
+  return r;
+}
+
+__device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
   asm volatile(
       "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
       "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-__device__ __forceinline__ uint32_t ldg_nc(const uint32_t* p) {
-  uint32_t v;
-  asm volatile("ld.global.nc.L1::no_allocate.u32 %0, [%1];" : "=r"(v) : "l"(p));
-  return v;
+// 16-byte global -> shared copy; bytes beyond src_bytes (0 or 16) are zero-filled.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+               "r"(src_bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
 __device__ __forceinline__ uint32_t half_scale_bf16x2(float s) {
@@ -76,107 +107,194 @@ __device__ __forceinline__ int find_mat(const DecodeBatch& b, int u) {
 }
 
 template <bool kTwoTiles>
-__global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_constant__ DecodeBatch b) {
+__global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_constant__ DecodeBatch b) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ int next_unit;
+  __shared__ int queue[kWarps][kQueue];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) &
+                                             ~static_cast<uintptr_t>(127));
+  const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int g = lane >> 2, t = lane & 3;
-  const int gwarp = static_cast<int>((blockIdx.x * kThreads + threadIdx.x) >> 5);
-  const int nwarps = static_cast<int>((gridDim.x * kThreads) >> 5);
   const int m = b.m;
+  const int uend = b.cta_unit[blockIdx.x + 1];
+  if (threadIdx.x == 0) next_unit = b.cta_unit[blockIdx.x];
+  __syncthreads();
+  uint8_t* ring = smem + warp * kDepth * kChunkBytes;
+  const uint32_t ring_u32 = static_cast<uint32_t>(__cvta_generic_to_shared(ring));
+  int* q = queue[warp];
+  uint32_t mul[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) mul[j] = opaque(1u << (14 - 2 * j));
 
-  for (int u = gwarp; u < b.total_units; u += nwarps) {
+  // ------------------------------------------------------------ prefetch cursor
+  // Lane l copies 16 bytes per chunk: row l / 2 of the unit, words 4 (l & 1) .. + 3.
+  const int crow = lane >> 1, chalf = lane & 1;
+  int qtail = 0;            // units claimed (queue writes)
+  int pu = -1;              // unit being prefetched (-1: stream exhausted)
+  int pc = 0, pnc = 0;      // its next chunk / chunk count
+  const uint32_t* psrc = nullptr;
+  bool prow = false;        // this lane's row exists
+  bool phalf = false;       // this lane's half of the last chunk lies past k
+  auto claim = [&]() {
+    int u = 0;
+    if (lane == 0) u = atomicAdd(&next_unit, 1);
+    u = __shfl_sync(0xffffffffu, u, 0);
+    if (u >= uend) {
+      pu = -1;
+      return;
+    }
+    const int d = find_mat(b, u);
+    const DecodeMat& mat = b.mats[d];
+    const int64_t row = static_cast<int64_t>(u - mat.unit0) * 16 + crow;
+    pu = u;
+    pc = 0;
+    pnc = static_cast<int>((mat.k + 127) >> 7);
+    prow = row < mat.n;
+    phalf = chalf && (mat.k & 127);
+    psrc = mat.codes + (prow ? row : 0) * (mat.k >> 4) + chalf * 4;
+    if (lane == 0) q[qtail % kQueue] = u;
+    ++qtail;
+  };
+  auto issue = [&](int slot) {
+    if (pu >= 0) {
+      const bool in = prow && !(phalf && pc + 1 == pnc);
+      cp_async16(ring_u32 + slot * kChunkBytes + crow * 32 + chalf * 16, psrc + 8 * pc,
+                 in ? 16u : 0u);
+      if (++pc == pnc) claim();
+    }
+    cp_async_commit();  // one group per slot, empty past the end of the stream
+  };
+
+  claim();
+  for (int s = 0; s < kDepth - 1; ++s) issue(s);
+
+  // ------------------------------------------------------------ consumer
+  int qhead = 0;
+  int slot = 0;
+  while (qhead < qtail) {
+    __syncwarp();
+    const int u = q[qhead % kQueue];
+    ++qhead;
     const int d = find_mat(b, u);
     const DecodeMat& mat = b.mats[d];
     const int64_t n = mat.n, k = mat.k;
     const int64_t r0 = static_cast<int64_t>(u - mat.unit0) * 16;
-    const int64_t words = k >> 4;                  // code words per row
-    const int nchunk = static_cast<int>(k >> 6);   // 64-wide chunks
-    const int64_t ra = r0 + g, rb = r0 + g + 8;    // this lane's two rows
+    const int64_t ra = r0 + g, rb = r0 + g + 8;
     const bool va = ra < n, vb = rb < n;
-    const uint32_t* ca = mat.codes + ra * words + t;
-    const uint32_t* cb = mat.codes + rb * words + t;
     const int log2g = mat.log2g;
     const int64_t gpr = k >> log2g;
-    const float* sa = mat.scales + ra * gpr;
-    const float* sb = mat.scales + rb * gpr;
-    // x rows of this lane's tokens (g and g + 8); tokens >= m read as zeros
-    const __nv_bfloat16* xa = static_cast<const __nv_bfloat16*>(mat.x) + static_cast<int64_t>(g) * k + 16 * t;
-    const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(mat.x) + static_cast<int64_t>(g + 8) * k + 16 * t;
+    const float* sa = mat.scales + (va ? ra : 0) * gpr;
+    const float* sb = mat.scales + (vb ? rb : 0) * gpr;
     const bool ta = g < m, tb = kTwoTiles && (g + 8 < m);
-
-    // code words of the first chunks
-    uint32_t qa[kPrefetch], qb[kPrefetch];
-#pragma unroll
-    for (int p = 0; p < kPrefetch; ++p) {
-      qa[p] = (va && p < nchunk) ? ldg_nc(ca + 4 * p) : 0u;
-      qb[p] = (vb && p < nchunk) ? ldg_nc(cb + 4 * p) : 0u;
-    }
-
+    const uint4* xa = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(mat.x) +
+                                                     static_cast<int64_t>(ta ? g : 0) * k + 32 * t);
+    const uint4* xb = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(mat.x) +
+                                                     static_cast<int64_t>(tb ? g + 8 : 0) * k + 32 * t);
+    const int nc = static_cast<int>((k + 127) >> 7);
+    // a lane's 32 offsets of the last chunk lie past k when k % 128 == 64 and t >= 2
+    const bool tail_lane = (k & 127) && t >= 2;
     float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
-    float part0[4] = {0.f, 0.f, 0.f, 0.f}, part1[4] = {0.f, 0.f, 0.f, 0.f};
-    const int chunks_per_group = log2g >= 6 ? (1 << (log2g - 6)) : 1;
+    float p0[4] = {0.f, 0.f, 0.f, 0.f}, p1[4] = {0.f, 0.f, 0.f, 0.f};
+    float q0[4] = {0.f, 0.f, 0.f, 0.f}, q1[4] = {0.f, 0.f, 0.f, 0.f};
 
-    for (int c0 = 0; c0 < nchunk; c0 += kPrefetch) {
+    if (log2g >= 7) {
+      // exact path: one scale per row per group of (g / 128) chunks
+      const int cpg = 1 << (log2g - 7);
+      int left = cpg;
+      int gi = 0;
+      for (int c = 0; c < nc; ++c) {
+        issue((slot + kDepth - 1) % kDepth);
+        cp_async_wait<kDepth - 1>();
+        __syncwarp();
+        const uint8_t* st = ring + slot * kChunkBytes;
+        const uint2 wa = *reinterpret_cast<const uint2*>(st + g * 32 + 8 * t);
+        const uint2 wb = *reinterpret_cast<const uint2*>(st + (g + 8) * 32 + 8 * t);
+        uint4 xv[4], yv[4];
 #pragma unroll
-      for (int p = 0; p < kPrefetch; ++p) {
-        const int c = c0 + p;
-        if (c >= nchunk) break;
-        const uint32_t wa = qa[p], wb = qb[p];
-        const int cn = c + kPrefetch;  // refill this slot
-        qa[p] = (va && cn < nchunk) ? ldg_nc(ca + 4 * cn) : 0u;
-        qb[p] = (vb && cn < nchunk) ? ldg_nc(cb + 4 * cn) : 0u;
-        // x fragments: 32 contiguous bytes per token row
-        uint4 x0 = make_uint4(0, 0, 0, 0), x1 = make_uint4(0, 0, 0, 0);
-        uint4 y0 = make_uint4(0, 0, 0, 0), y1 = make_uint4(0, 0, 0, 0);
-        if (ta) {
-          x0 = __ldg(reinterpret_cast<const uint4*>(xa + 64 * c));
-          x1 = __ldg(reinterpret_cast<const uint4*>(xa + 64 * c + 8));
+        for (int i = 0; i < 4; ++i) {
+          xv[i] = ta ? __ldg(xa + 16 * c + i) : make_uint4(0, 0, 0, 0);
+          if (kTwoTiles) yv[i] = tb ? __ldg(xb + 16 * c + i) : make_uint4(0, 0, 0, 0);
         }
-        if (tb) {
-          y0 = __ldg(reinterpret_cast<const uint4*>(xb + 64 * c));
-          y1 = __ldg(reinterpret_cast<const uint4*>(xb + 64 * c + 8));
+        const uint32_t* xr = reinterpret_cast<const uint32_t*>(xv);
+        const uint32_t* yr = reinterpret_cast<const uint32_t*>(yv);
+#pragma unroll
+        for (int kb = 0; kb < 8; ++kb) {
+          const uint32_t ua = kb < 4 ? wa.x : wa.y, ub = kb < 4 ? wb.x : wb.y;
+          const int j = 2 * (kb & 3);
+          const uint32_t a0 = pair_bits(ua, j, mul[j]), a1 = pair_bits(ub, j, mul[j]);
+          const uint32_t a2 = pair_bits(ua, j + 1, mul[j + 1]), a3 = pair_bits(ub, j + 1, mul[j + 1]);
+          if (kb & 1) {
+            mma16816(q0, a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
+            if (kTwoTiles) mma16816(q1, a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
+          } else {
+            mma16816(p0, a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
+            if (kTwoTiles) mma16816(p1, a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
+          }
         }
-        const uint32_t xr[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-        const uint32_t yr[8] = {y0.x, y0.y, y0.z, y0.w, y1.x, y1.y, y1.z, y1.w};
-        if (log2g == 5) {
-          // g = 32: lane t's offsets 16t..16t+15 lie in group (64c + 16t) / 32
-          const int64_t gi = (static_cast<int64_t>(c) * 64 + 16 * t) >> 5;
-          const uint32_t ha = va ? half_scale_bf16x2(__ldg(sa + gi)) : 0u;
-          const uint32_t hb = vb ? half_scale_bf16x2(__ldg(sb + gi)) : 0u;
+        __syncwarp();
+        slot = slot + 1 == kDepth ? 0 : slot + 1;
+        if (--left == 0) {
+          // group closed: acc += (s / 2) * partial; rows g (slots 0, 1), g + 8 (2, 3)
+          left = cpg;
+          const float ha = va ? 0.5f * __ldg(sa + gi) : 0.f;
+          const float hb = vb ? 0.5f * __ldg(sb + gi) : 0.f;
+          ++gi;
 #pragma unroll
-          for (int kb = 0; kb < 4; ++kb) {
-            const uint32_t a[4] = {bmul2(pair_bits(wa, 2 * kb), ha), bmul2(pair_bits(wb, 2 * kb), hb),
-                                   bmul2(pair_bits(wa, 2 * kb + 1), ha),
-                                   bmul2(pair_bits(wb, 2 * kb + 1), hb)};
-            mma16816(acc0, a, xr[2 * kb], xr[2 * kb + 1]);
-            if (kTwoTiles) mma16816(acc1, a, yr[2 * kb], yr[2 * kb + 1]);
-          }
-        } else {
-#pragma unroll
-          for (int kb = 0; kb < 4; ++kb) {
-            const uint32_t a[4] = {pair_bits(wa, 2 * kb), pair_bits(wb, 2 * kb),
-                                   pair_bits(wa, 2 * kb + 1), pair_bits(wb, 2 * kb + 1)};
-            mma16816(part0, a, xr[2 * kb], xr[2 * kb + 1]);
-            if (kTwoTiles) mma16816(part1, a, yr[2 * kb], yr[2 * kb + 1]);
-          }
-          if ((c + 1) % chunks_per_group == 0) {
-            // close the group: acc += (s / 2) * partial, rows g (slots 0,1) and g+8 (2,3)
-            const int64_t gi = (static_cast<int64_t>(c) * 64) >> log2g;
-            const float ha = va ? 0.5f * __ldg(sa + gi) : 0.f;
-            const float hb = vb ? 0.5f * __ldg(sb + gi) : 0.f;
-            acc0[0] = fmaf(ha, part0[0], acc0[0]);
-            acc0[1] = fmaf(ha, part0[1], acc0[1]);
-            acc0[2] = fmaf(hb, part0[2], acc0[2]);
-            acc0[3] = fmaf(hb, part0[3], acc0[3]);
-            part0[0] = part0[1] = part0[2] = part0[3] = 0.f;
+          for (int i = 0; i < 4; ++i) {
+            const float h = i < 2 ? ha : hb;
+            acc0[i] = fmaf(h, p0[i] + q0[i], acc0[i]);
+            p0[i] = q0[i] = 0.f;
             if (kTwoTiles) {
-              acc1[0] = fmaf(ha, part1[0], acc1[0]);
-              acc1[1] = fmaf(ha, part1[1], acc1[1]);
-              acc1[2] = fmaf(hb, part1[2], acc1[2]);
-              acc1[3] = fmaf(hb, part1[3], acc1[3]);
-              part1[0] = part1[1] = part1[2] = part1[3] = 0.f;
+              acc1[i] = fmaf(h, p1[i] + q1[i], acc1[i]);
+              p1[i] = q1[i] = 0.f;
             }
           }
         }
+      }
+    } else {
+      // g = 32 or 64: lane t's offsets 32t .. 32t + 31 of a chunk lie in one group
+      const int gshift = 7 - log2g;  // groups per chunk = 1 << gshift
+      for (int c = 0; c < nc; ++c) {
+        issue((slot + kDepth - 1) % kDepth);
+        cp_async_wait<kDepth - 1>();
+        __syncwarp();
+        const bool kin = !(tail_lane && c + 1 == nc);
+        const uint8_t* st = ring + slot * kChunkBytes;
+        const uint2 wa = *reinterpret_cast<const uint2*>(st + g * 32 + 8 * t);
+        const uint2 wb = *reinterpret_cast<const uint2*>(st + (g + 8) * 32 + 8 * t);
+        const int64_t gi = (static_cast<int64_t>(c) << gshift) + (t >> (log2g - 5));
+        const uint32_t ha = (va && kin) ? half_scale_bf16x2(__ldg(sa + gi)) : 0u;
+        const uint32_t hb = (vb && kin) ? half_scale_bf16x2(__ldg(sb + gi)) : 0u;
+        uint4 xv[4], yv[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          xv[i] = (ta && kin) ? __ldg(xa + 16 * c + i) : make_uint4(0, 0, 0, 0);
+          if (kTwoTiles) yv[i] = (tb && kin) ? __ldg(xb + 16 * c + i) : make_uint4(0, 0, 0, 0);
+        }
+        const uint32_t* xr = reinterpret_cast<const uint32_t*>(xv);
+        const uint32_t* yr = reinterpret_cast<const uint32_t*>(yv);
+#pragma unroll
+        for (int kb = 0; kb < 8; ++kb) {
+          const uint32_t ua = kb < 4 ? wa.x : wa.y, ub = kb < 4 ? wb.x : wb.y;
+          const int j = 2 * (kb & 3);
+          const uint32_t a0 = bmul2(pair_bits(ua, j, mul[j]), ha), a1 = bmul2(pair_bits(ub, j, mul[j]), hb);
+          const uint32_t a2 = bmul2(pair_bits(ua, j + 1, mul[j + 1]), ha), a3 = bmul2(pair_bits(ub, j + 1, mul[j + 1]), hb);
+          if (kb & 1) {
+            mma16816(q0, a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
+            if (kTwoTiles) mma16816(q1, a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
+          } else {
+            mma16816(acc0, a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
+            if (kTwoTiles) mma16816(acc1, a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
+          }
+        }
+        __syncwarp();
+        slot = slot + 1 == kDepth ? 0 : slot + 1;
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        acc0[i] += q0[i];
+        if (kTwoTiles) acc1[i] += q1[i];
       }
     }
 
@@ -200,20 +318,50 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
       store(8 + 2 * t + 1, rb, acc1[3]);
     }
   }
+  cp_async_wait<0>();  // nothing may still write this warp's ring when it exits
 }
 
 }  // namespace
 
-cudaError_t launch_decode(const DecodeBatch& b, int num_sms, cudaStream_t stream) {
+cudaError_t launch_decode(DecodeBatch& b, int num_sms, cudaStream_t stream) {
   if (b.total_units <= 0) return cudaSuccess;
-  const int warps_per_block = kThreads / 32;
-  int64_t blocks = (static_cast<int64_t>(b.total_units) + warps_per_block - 1) / warps_per_block;
-  const int64_t cap = static_cast<int64_t>(num_sms) * 3;
-  if (blocks > cap) blocks = cap;
-  if (b.m > 8)
-    decode_kernel<true><<<static_cast<unsigned>(blocks), kThreads, 0, stream>>>(b);
-  else
-    decode_kernel<false><<<static_cast<unsigned>(blocks), kThreads, 0, stream>>>(b);
+  int64_t blocks = (static_cast<int64_t>(b.total_units) + kWarps - 1) / kWarps;
+  if (blocks > num_sms) blocks = num_sms;
+  if (blocks > kDecodeMaxCtas) blocks = kDecodeMaxCtas;
+  // Split the units into `blocks` contiguous ranges of about equal chunk count.
+  int64_t work = 0;
+  for (int d = 0; d < b.count; ++d) {
+    const int64_t units = (b.mats[d].n + 15) / 16;
+    work += units * ((b.mats[d].k + 127) / 128);
+  }
+  int c = 0;
+  int64_t acc = 0;
+  b.cta_unit[0] = 0;
+  for (int d = 0; d < b.count && c + 1 < blocks; ++d) {
+    const int64_t units = (b.mats[d].n + 15) / 16;
+    const int64_t per = (b.mats[d].k + 127) / 128;
+    for (int64_t u = 0; u < units && c + 1 < blocks; ++u) {
+      acc += per;
+      // close range c once it holds its share (c + 1) * work / blocks
+      while (c + 1 < blocks && acc * blocks >= (c + 1) * work) {
+        b.cta_unit[++c] = b.mats[d].unit0 + static_cast<int32_t>(u) + 1;
+      }
+    }
+  }
+  while (c < blocks) b.cta_unit[++c] = b.total_units;
+  const size_t smem = kSmemBytes + 128;
+  cudaError_t e;
+  if (b.m > 8) {
+    e = cudaFuncSetAttribute(decode_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    decode_kernel<true><<<static_cast<unsigned>(blocks), kThreads, smem, stream>>>(b);
+  } else {
+    e = cudaFuncSetAttribute(decode_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    decode_kernel<false><<<static_cast<unsigned>(blocks), kThreads, smem, stream>>>(b);
+  }
   return cudaGetLastError();
 }
 

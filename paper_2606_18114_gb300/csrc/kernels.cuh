@@ -53,16 +53,19 @@ struct DecodeMat {
 };
 
 constexpr int kDecodeMaxMats = 256;
+constexpr int kDecodeMaxCtas = 256;
 
 struct DecodeBatch {
   DecodeMat mats[kDecodeMaxMats];
+  int32_t cta_unit[kDecodeMaxCtas + 1];  // CTA c owns units [cta_unit[c], cta_unit[c + 1])
+  int* status;            // device status word (timeouts)
   int32_t count;
   int32_t m;              // tokens, 1..16
   int32_t total_units;    // sum over matrices of ceil(n / 16)
   int32_t pad;
 };
 
-cudaError_t launch_decode(const DecodeBatch& batch, int num_sms, cudaStream_t stream);
+cudaError_t launch_decode(DecodeBatch& batch, int num_sms, cudaStream_t stream);
 
 // dw_gemm.cu -----------------------------------------------------------------
 // dW[n][k] (+)= sum_m dy[m][n] x[m][k], both operands MN-major from TMA.

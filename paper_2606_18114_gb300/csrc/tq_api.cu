@@ -216,6 +216,7 @@ tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
     if (units >= (int64_t(1) << 31)) return fail(TQ_ERR_UNSUPPORTED, "too many decode rows");
   }
   if (used == 0) return TQ_OK;
+  b.status = dev->status;
   b.count = used;
   b.m = static_cast<int32_t>(m);
   b.total_units = static_cast<int32_t>(units);

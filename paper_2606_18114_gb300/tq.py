@@ -19,6 +19,7 @@ __all__ = [
     "linear_fwd",
     "linear_bwd",
     "linear_fwd_batched",
+    "fwd_batch",
     "device_status",
     "version",
     "OUT_F32",
@@ -170,15 +171,22 @@ def linear_bwd(dy: torch.Tensor, x: Optional[torch.Tensor], codes: torch.Tensor,
     return dx, dw
 
 
-def linear_fwd_batched(items: Sequence[dict], m: int, stream=None) -> None:
-    """Decode forward over many matrices in one call.
+def fwd_batch(items: Sequence[dict]):
+    """Descriptor array for ``linear_fwd_batched`` (build once, call many times).
 
     ``items``: dicts with ``x, codes, scales, y, g`` (tensors already allocated,
-    ``y`` written in place).
+    ``y`` written in place). The tensors must outlive the array's use.
     """
     arr = (FwdDesc * len(items))()
     for i, it in enumerate(items):
         codes = it["codes"]
         arr[i] = FwdDesc(_ptr(it["x"]), _ptr(codes), _ptr(it["scales"]), _ptr(it["y"]),
                          codes.shape[0], codes.shape[1] * 16, it["g"], _out_code(it["y"].dtype))
-    _check(load().tq_linear_fwd_batched(arr, len(items), m, _stream(stream)))
+    return arr
+
+
+def linear_fwd_batched(items, m: int, stream=None) -> None:
+    """Decode forward over many matrices in one call (``items`` as for ``fwd_batch``,
+    or an array that ``fwd_batch`` returned)."""
+    arr = items if isinstance(items, ctypes.Array) else fwd_batch(items)
+    _check(load().tq_linear_fwd_batched(arr, len(arr), m, _stream(stream)))
