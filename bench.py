@@ -41,7 +41,8 @@ G = 128
 N_LAYERS = 48
 METRIC = "W1.58A16 linear fwd+bwd TFLOP/s"
 WORKLOAD = ("Mamba-2 1.3B in_proj prefill, one step = tq_quantize W[8512,2048] (g=128) + "
-            "tq_linear_fwd + tq_linear_bwd (dX, dW) at M=16384 (batch 8 x seq 2048)")
+            "tq_codes_transpose + tq_linear_fwd + tq_linear_bwd (dX, dW) at M=16384 "
+            "(batch 8 x seq 2048)")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -162,6 +163,7 @@ class Prefill:
         self.x = torch.randn((m, k), generator=gen, device="cuda").to(torch.bfloat16)
         self.dy = (torch.randn((m, n), generator=gen, device="cuda") * 1e-2).to(torch.bfloat16)
         self.codes = torch.empty((n, k // 16), dtype=torch.int32, device="cuda")
+        self.codes_t = torch.empty((k, 4 * ((n + 63) // 64)), dtype=torch.int32, device="cuda")
         self.s = torch.empty((n, k // g), dtype=torch.float32, device="cuda")
         self.z = torch.empty((n, k // g), dtype=torch.int32, device="cuda")
         self.y = torch.empty((m, n), dtype=torch.float32, device="cuda")
@@ -182,21 +184,24 @@ class Prefill:
         rec(0)
         tq.quantize(self.w, self.g, out=(self.codes, self.s, self.z))
         rec(1)
-        tq.linear_fwd(self.x, self.codes, self.s, self.g, y=self.y)
+        tq.codes_transpose(self.codes, self.k, out=self.codes_t)
         rec(2)
-        tq.linear_bwd(self.dy, self.x, self.codes, self.s, self.k, self.g, want_dw=False,
-                      dx=self.dx)
+        tq.linear_fwd(self.x, self.codes, self.s, self.g, y=self.y)
         rec(3)
+        tq.linear_bwd(self.dy, self.x, self.codes, self.s, self.k, self.g, want_dw=False,
+                      dx=self.dx, codes_t=self.codes_t)
+        rec(4)
         tq.linear_bwd(self.dy, self.x, self.codes, self.s, self.k, self.g, want_dx=False,
                       dw=self.dw)
-        rec(4)
+        rec(5)
 
 
 KERNELS = [  # name, source files, event span
     ("quantize", ["quantize.cu"], (0, 1)),
-    ("fwd", ["ts_gemm.cu", "ptx.cuh"], (1, 2)),
-    ("dx", ["ts_gemm.cu", "ptx.cuh"], (2, 3)),
-    ("dw", ["dw_gemm.cu", "ptx.cuh"], (3, 4)),
+    ("transpose", ["quantize.cu"], (1, 2)),
+    ("fwd", ["ts_gemm.cu", "ptx.cuh"], (2, 3)),
+    ("dx", ["ts_gemm.cu", "ptx.cuh"], (3, 4)),
+    ("dw", ["dw_gemm.cu", "ptx.cuh"], (4, 5)),
 ]
 
 
@@ -204,7 +209,7 @@ def time_prefill(p: Prefill, steps, warmup, world):
     for _ in range(warmup):
         p.step()
     torch.cuda.synchronize()
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(steps)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(steps)]
     barrier(world)
     torch.cuda.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
@@ -417,10 +422,13 @@ def run_only(args):
         return
     p = Prefill(tq, IN_PROJ[0], IN_PROJ[1], M_PREFILL, G, seed=7)
     tq.quantize(p.w, p.g, out=(p.codes, p.s, p.z))
+    tq.codes_transpose(p.codes, p.k, out=p.codes_t)
     calls = {
         "quantize": lambda: tq.quantize(p.w, p.g, out=(p.codes, p.s, p.z)),
+        "transpose": lambda: tq.codes_transpose(p.codes, p.k, out=p.codes_t),
         "fwd": lambda: tq.linear_fwd(p.x, p.codes, p.s, p.g, y=p.y),
-        "dx": lambda: tq.linear_bwd(p.dy, p.x, p.codes, p.s, p.k, p.g, want_dw=False, dx=p.dx),
+        "dx": lambda: tq.linear_bwd(p.dy, p.x, p.codes, p.s, p.k, p.g, want_dw=False, dx=p.dx,
+                                    codes_t=p.codes_t),
         "dw": lambda: tq.linear_bwd(p.dy, p.x, p.codes, p.s, p.k, p.g, want_dx=False, dw=p.dw),
     }
     fn = calls[args.only]
@@ -448,7 +456,7 @@ def main():
     ap.add_argument("--impl", default="tq", choices=["tq", "reference"])
     ap.add_argument("--no-extra", action="store_true", help="skip decode/quantize sweeps")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
-    ap.add_argument("--only", choices=["quantize", "fwd", "dx", "dw", "decode"],
+    ap.add_argument("--only", choices=["quantize", "transpose", "fwd", "dx", "dw", "decode"],
                     help="profiling aid: run just this kernel of the step (or the batched "
                          "M=1 decode) --warmup + --steps times and print its time")
     args = ap.parse_args()
@@ -478,15 +486,16 @@ def main():
     kinfo = {}
     for name, files, _ in KERNELS:
         t = per[name]
-        if name == "quantize":
-            ach = p.quantize_bytes() / (t * 1e-3) / 1e9
+        if name in ("quantize", "transpose"):
+            nbytes = p.quantize_bytes() if name == "quantize" else 2 * p.n * p.k // 4
+            ach = nbytes / (t * 1e-3) / 1e9
             kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "GB/s",
                            "frac": round(ach / pk["hbm_gbs"], 4)}
         else:
             ach = gemm_flops / (t * 1e-3) / 1e12
             kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "TFLOP/s",
                            "frac": round(ach / pk["bf16_tflops"], 4)}
-    dom = max((n for n, _, _ in KERNELS if n != "quantize"), key=lambda n: per[n])
+    dom = max((n for n, _, _ in KERNELS if n not in ("quantize", "transpose")), key=lambda n: per[n])
     dom_files = dict((n, f) for n, f, _ in KERNELS)[dom]
     roof = {"kernel": dom, "bound": "tensor", "achieved": kinfo[dom]["achieved"],
             "peak": pk["bf16_tflops"], "unit": "TFLOP/s", "frac": kinfo[dom]["frac"],
@@ -510,7 +519,7 @@ def main():
         "e2e": {"value": round(world * p.flops / (e2e_ms * 1e-3) / 1e12, 2), "unit": "TFLOP/s",
                 "ms_per_step": round(e2e_ms, 3), "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
-        "gpu_launches": 4 * args.steps,
+        "gpu_launches": len(KERNELS) * args.steps,
         "clocks": clk.summary(),
     }
     if not args.no_extra and rank == 0:

@@ -107,12 +107,29 @@ TQ_API tq_status tq_linear_fwd(const void* x, int64_t m, int64_t k,
  *   dx           out: [m][k], fp32 or bf16 (dx_dtype); NULL skips dX.
  *   dw           out: fp32 [n][k]; NULL skips dW. accumulate_dw != 0 adds to
  *                dw instead of overwriting it.
+ *   codes_t      optional: tq_codes_transpose's output for the same codes. With it
+ *                dX expands the codes of W^T like the forward expands W's (faster);
+ *                NULL makes dX read `codes` directly.
  *   Requires k % 64 == 0, k % g == 0, n % 8 == 0. x may be NULL when dw is.
  */
 TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t n, int64_t k,
-                        const uint32_t* codes, const float* scales, int32_t g,
-                        void* dx, int32_t dx_dtype, float* dw, int32_t accumulate_dw,
-                        void* stream);
+                        const uint32_t* codes, const uint32_t* codes_t, const float* scales,
+                        int32_t g, void* dx, int32_t dx_dtype, float* dw,
+                        int32_t accumulate_dw, void* stream);
+
+/*
+ * tq_codes_transpose — the packed codes of W^T, a re-layout of tq_quantize's codes
+ * (no arithmetic of the method) that the STE dX product streams along its
+ * reduction (n):
+ *   codes        uint32 [n][k/16], layout above.
+ *   codes_t      out: uint32 [k][ldt] with ldt = 4 * ceil(n / 64) words per row;
+ *                word w of row k holds the codes of (n', k) for n' in
+ *                [16w, 16w + 16) at the bit of i = n' % 16 (same rule as codes);
+ *                codes past n are 0.
+ *   Requires k % 16 == 0.
+ */
+TQ_API tq_status tq_codes_transpose(const uint32_t* codes, int64_t n, int64_t k,
+                                    uint32_t* codes_t, void* stream);
 
 /* One matrix of a batched decode call (tq_linear_fwd_batched). */
 typedef struct {

@@ -11,14 +11,19 @@ namespace tq {
 cudaError_t launch_quantize(const float* w, int64_t n, int64_t k, int g, uint32_t* codes,
                             float* scales, int32_t* zeros, int num_sms, cudaStream_t stream);
 
+// codes [n][k/16] -> codes_t [k][4 * ceil(n / 64)] (the codes of W^T).
+cudaError_t launch_transpose_codes(const uint32_t* codes, int64_t n, int64_t k, uint32_t* codes_t,
+                                   cudaStream_t stream);
+
 // ts_gemm.cu -----------------------------------------------------------------
 // Ternary x bf16 products with the expanded ternary weights as the tensor-memory
 // A operand. kTsFwd: out[m][n] = sum_k x[m][k] w^[n][k] (B = x, rows = n).
-// kTsDx: out[m][k] = sum_n dy[m][n] w^[n][k] (B = dy, rows = k).
-enum TsMode : int { kTsFwd = 0, kTsDx = 1 };
+// kTsDx: out[m][k] = sum_n dy[m][n] w^[n][k] (B = dy, rows = k), codes read as is.
+// kTsDxT: the same product with the transposed codes (codes_t) as input.
+enum TsMode : int { kTsFwd = 0, kTsDx = 1, kTsDxT = 2 };
 
 struct TsArgs {
-  const uint32_t* codes;  // uint32 [wn][wk/16]
+  const uint32_t* codes;  // uint32 [wn][wk/16] (fwd, dx) or codes_t [wk][ldt] (dxt)
   const float* scales;    // fp32 [wn][wk/g]
   void* out;              // [m][rows], fp32 or bf16
   int* status;            // device status word (timeouts)

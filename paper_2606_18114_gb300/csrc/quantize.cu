@@ -109,7 +109,50 @@ cudaError_t launch(const float* w, int64_t total, uint32_t* codes, float* scales
   return cudaGetLastError();
 }
 
+// codes [n][k/16] -> codes_t [k][ldt]: a 128 x 128 (n x k) tile per block. The tile's
+// 128 rows x 8 code words are read with one 32-byte sector per row, and each
+// output row k receives 8 consecutive words (one sector) of the transposed tile.
+__device__ __forceinline__ int code_pos(int i) { return 16 * (i & 1) + 2 * (i >> 1); }
+
+__global__ void __launch_bounds__(256) transpose_codes_kernel(const uint32_t* __restrict__ codes,
+                                                              int64_t n, int64_t k,
+                                                              uint32_t* __restrict__ codes_t,
+                                                              int64_t ldt) {
+  __shared__ uint32_t tile[128][9];
+  const int64_t n0 = static_cast<int64_t>(blockIdx.y) * 128;
+  const int64_t k0 = static_cast<int64_t>(blockIdx.x) * 128;
+  const int64_t words = k >> 4;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int idx = threadIdx.x + 256 * i;
+    const int r = idx >> 3, c = idx & 7;
+    const int64_t row = n0 + r, col = (k0 >> 4) + c;
+    tile[r][c] = (row < n && col < words) ? codes[row * words + col] : 0u;
+  }
+  __syncthreads();
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int idx = threadIdx.x + 256 * i;
+    const int kk = idx >> 3, ww = idx & 7;
+    const int64_t kg = k0 + kk, wg = (n0 >> 4) + ww;
+    if (kg >= k || wg >= ldt) continue;
+    const int c = kk >> 4, sh = code_pos(kk & 15);
+    uint32_t out = 0;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) out |= ((tile[16 * ww + j][c] >> sh) & 3u) << code_pos(j);
+    codes_t[kg * ldt + wg] = out;
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_transpose_codes(const uint32_t* codes, int64_t n, int64_t k, uint32_t* codes_t,
+                                   cudaStream_t stream) {
+  const int64_t ldt = 4 * ((n + 63) / 64);
+  dim3 grid(static_cast<unsigned>((k + 127) / 128), static_cast<unsigned>((n + 127) / 128));
+  transpose_codes_kernel<<<grid, 256, 0, stream>>>(codes, n, k, codes_t, ldt);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_quantize(const float* w, int64_t n, int64_t k, int g, uint32_t* codes,
                             float* scales, int32_t* zeros, int num_sms, cudaStream_t stream) {

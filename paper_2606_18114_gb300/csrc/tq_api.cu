@@ -301,9 +301,26 @@ TQ_API tq_status tq_linear_fwd_batched(const tq_fwd_desc* descs, int32_t count, 
   return decode_checked(descs, count, m, static_cast<cudaStream_t>(stream));
 }
 
+TQ_API tq_status tq_codes_transpose(const uint32_t* codes, int64_t n, int64_t k,
+                                    uint32_t* codes_t, void* stream) {
+  g_err[0] = 0;
+  if (n < 0 || k < 0) return fail(TQ_ERR_INVALID_ARG, "negative size");
+  if (k % 16 != 0) return fail(TQ_ERR_INVALID_ARG, "k=%lld is not a multiple of 16", (long long)k);
+  if (n == 0 || k == 0) return TQ_OK;
+  if (n > kMaxDim || k > kMaxDim || (n + 127) / 128 > 65535)
+    return fail(TQ_ERR_UNSUPPORTED, "dimension too large");
+  TQ_TRY(check_ptr(codes, "codes"));
+  TQ_TRY(check_ptr(codes_t, "codes_t"));
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaError_t e = tq::launch_transpose_codes(codes, n, k, codes_t, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "transpose launch");
+}
+
 TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t n, int64_t k,
-                               const uint32_t* codes, const float* scales, int32_t g, void* dx,
-                               int32_t dx_dtype, float* dw, int32_t accumulate_dw, void* stream) {
+                               const uint32_t* codes, const uint32_t* codes_t,
+                               const float* scales, int32_t g, void* dx, int32_t dx_dtype,
+                               float* dw, int32_t accumulate_dw, void* stream) {
   g_err[0] = 0;
   TQ_TRY(check_linear_shape(m, n, k, g));
   if (n % 8 != 0)
@@ -317,7 +334,8 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
     TQ_TRY(check_ptr(dx, "dx"));
     if (n > 0) {
       TQ_TRY(check_ptr(dy, "dy"));
-      TQ_TRY(check_ptr(codes, "codes"));
+      if (codes_t == nullptr) TQ_TRY(check_ptr(codes, "codes"));
+      else TQ_TRY(check_ptr(codes_t, "codes_t"));
       TQ_TRY(check_ptr(scales, "scales"));
     }
   }
@@ -345,10 +363,15 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
       CUtensorMap tb, tc;
       TQ_TRY(make_map(&tb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, dy, n, m, 64, bn,
                       CU_TENSOR_MAP_SWIZZLE_128B));
-      TQ_TRY(make_map(&tc, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, codes, k / 16, n, 8, 128,
-                      CU_TENSOR_MAP_SWIZZLE_NONE));
+      const int64_t ldt = 4 * ((n + 63) / 64);  // codes_t row length (words)
+      if (codes_t != nullptr)
+        TQ_TRY(make_map(&tc, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, codes_t, ldt, k, 8, 128,
+                        CU_TENSOR_MAP_SWIZZLE_NONE));
+      else
+        TQ_TRY(make_map(&tc, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, codes, k / 16, n, 8, 128,
+                        CU_TENSOR_MAP_SWIZZLE_NONE));
       tq::TsArgs a{};
-      a.codes = codes;
+      a.codes = codes_t != nullptr ? codes_t : codes;
       a.scales = scales;
       a.out = dx;
       a.status = dev->status;
@@ -357,7 +380,8 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
       a.m = m;
       a.log2g = log2_group(g);
       a.out_bf16 = dx_dtype == TQ_OUT_BF16;
-      cudaError_t e = tq::launch_ts_gemm(tq::kTsDx, bn, tb, tc, a, dev->num_sms, st);
+      cudaError_t e = tq::launch_ts_gemm(codes_t != nullptr ? tq::kTsDxT : tq::kTsDx, bn, tb, tc,
+                                         a, dev->num_sms, st);
       if (e != cudaSuccess) return cuda_fail(e, "dX launch");
     }
   }

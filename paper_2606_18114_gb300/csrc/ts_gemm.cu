@@ -183,7 +183,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_2d(stage, &tmap_b, full_bar(s), kb * kKBlock, static_cast<int32_t>(m0));
         tma_load_2d(stage + L::kSubBytes, &tmap_b, full_bar(s), kb * kKBlock + 64,
                     static_cast<int32_t>(m0));
-        if (MODE == kTsFwd)
+        if (MODE != kTsDx)  // codes (forward) or codes_t (dX): rows = this tile's rows
           tma_load_2d(stage + L::kBBytes, &tmap_codes, full_bar(s), kb * (kKBlock / 16),
                       static_cast<int32_t>(r0));
         else
@@ -351,7 +351,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     } else {
       // dX: this thread is input feature k = row; a warp shares one k-group, and
-      // warpgroup wg covers rows n in [kb*128 + 64 wg, kb*128 + 64 wg + 64).
+      // warpgroup wg covers rows n in [kb*128 + 64 wg, kb*128 + 64 wg + 64). The
+      // scale varies along n: each warp stages the bf16(s)/2 of its 64 rows n in
+      // shared memory and reads them as pairs.
       auto load_sc = [&](const Cursor& c) -> float2 {
         float2 r = make_float2(0.f, 0.f);
         const int64_t kwarp = c.r0 + quad * 32;
@@ -363,15 +365,46 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (n_b < args.wn) r.y = __ldg(args.scales + n_b * gpr + gk);
         return r;
       };
+      __nv_bfloat16* sbuf =
+          reinterpret_cast<__nv_bfloat16*>(smem + L::kScaleOff) + (wg * 4 + quad) * 128;
+      float2 p0 = load_sc(cur), p1 = load_sc(cursor_at(1));
+      if (MODE == kTsDxT) {
+        // codes_t: this thread's row k of the transposed codes holds rows n along it,
+        // so the expansion is the forward's with a scale pair per pair of rows n.
+        for (; cur.it < total; advance(cur), advance(pre)) {
+          const int it = cur.it;
+          const int s = it % kSmem, as = it % kAS;
+          const float2 sc = p0;
+          p0 = p1;
+          p1 = load_sc(pre);
+          __nv_bfloat16* sb = sbuf + (it & 1) * 64;
+          sb[lane] = __float2bfloat16_rn(0.5f * sc.x);
+          sb[lane + 32] = __float2bfloat16_rn(0.5f * sc.y);
+          __syncwarp();
+          if (!warp_wait(full_bar(s), (it / kSmem) & 1, status)) break;
+          const uint4 cw = *reinterpret_cast<const uint4*>(smem + s * L::kStageBytes + L::kBBytes +
+                                                           r_local * 32 + wg * 16);
+          const uint4* sp = reinterpret_cast<const uint4*>(sb);  // 32 pairs of rows n
+          const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
+          uint32_t a[32];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const uint4 s0 = sp[2 * q], s1 = sp[2 * q + 1];
+            const uint32_t pr[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+              a[8 * q + j] = bmul2((words[q] << (14 - 2 * j)) & 0xC000C000u, pr[j]);
+          }
+          if (!a_free(it)) break;
+          publish(as, a);
+        }
+      } else {
       // this thread's 2-bit field inside a code word of its 16-wide k slice
       const int i16 = r_local & 15;
       const int pos = 16 * (i16 & 1) + 2 * (i16 >> 1);
       const uint32_t sel = static_cast<uint32_t>(((pos >> 3) << 4) | ((4 + (pos >> 3)) << 12));
       const int shift = 6 - (pos & 7);
       const int xw = r_local >> 4;
-      __nv_bfloat16* sbuf =
-          reinterpret_cast<__nv_bfloat16*>(smem + L::kScaleOff) + (wg * 4 + quad) * 128;
-      float2 p0 = load_sc(cur), p1 = load_sc(cursor_at(1));
       for (; cur.it < total; advance(cur), advance(pre)) {
         const int it = cur.it;
         const int s = it % kSmem, as = it % kAS;
@@ -396,6 +429,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (!a_free(it)) break;
         publish(as, a);
+      }
       }
     }
   }
@@ -436,9 +470,12 @@ cudaError_t launch_ts_gemm(int mode, int bn, const CUtensorMap& tb, const CUtens
                            const TsArgs& a, int num_sms, cudaStream_t stream) {
   if (mode == kTsFwd) {
     if (bn == 192) return launch_impl<kTsFwd, 192>(tb, tc, a, num_sms, stream);
-  } else {
+  } else if (mode == kTsDx) {
     if (bn == 16) return launch_impl<kTsDx, 16>(tb, tc, a, num_sms, stream);
     if (bn == 256) return launch_impl<kTsDx, 256>(tb, tc, a, num_sms, stream);
+  } else if (mode == kTsDxT) {
+    if (bn == 16) return launch_impl<kTsDxT, 16>(tb, tc, a, num_sms, stream);
+    if (bn == 256) return launch_impl<kTsDxT, 256>(tb, tc, a, num_sms, stream);
   }
   return cudaErrorInvalidValue;
 }

@@ -18,6 +18,7 @@ __all__ = [
     "quantize",
     "linear_fwd",
     "linear_bwd",
+    "codes_transpose",
     "linear_fwd_batched",
     "fwd_batch",
     "device_status",
@@ -32,8 +33,8 @@ OUT_BF16 = 1
 STATUS = {0: "TQ_OK", 1: "TQ_ERR_INVALID_ARG", 2: "TQ_ERR_UNSUPPORTED", 3: "TQ_ERR_CUDA",
           4: "TQ_ERR_TIMEOUT"}
 # Every symbol include/tq.h declares.
-EXPORTS = ("tq_quantize", "tq_linear_fwd", "tq_linear_bwd", "tq_linear_fwd_batched",
-           "tq_device_status", "tq_last_error", "tq_version")
+EXPORTS = ("tq_quantize", "tq_linear_fwd", "tq_linear_bwd", "tq_codes_transpose",
+           "tq_linear_fwd_batched", "tq_device_status", "tq_last_error", "tq_version")
 
 _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtq.so")
 _lib = None
@@ -70,11 +71,12 @@ def load(path: Optional[str] = None):
     i64, i32, vp = ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p
     lib.tq_quantize.argtypes = [vp, i64, i64, i32, vp, vp, vp, vp]
     lib.tq_linear_fwd.argtypes = [vp, i64, i64, vp, vp, i64, i32, vp, i32, vp]
-    lib.tq_linear_bwd.argtypes = [vp, vp, i64, i64, i64, vp, vp, i32, vp, i32, vp, i32, vp]
+    lib.tq_linear_bwd.argtypes = [vp, vp, i64, i64, i64, vp, vp, vp, i32, vp, i32, vp, i32, vp]
+    lib.tq_codes_transpose.argtypes = [vp, i64, i64, vp, vp]
     lib.tq_linear_fwd_batched.argtypes = [ctypes.POINTER(FwdDesc), i32, i64, vp]
     lib.tq_device_status.argtypes = [vp]
-    for name in ("tq_quantize", "tq_linear_fwd", "tq_linear_bwd", "tq_linear_fwd_batched",
-                 "tq_device_status"):
+    for name in ("tq_quantize", "tq_linear_fwd", "tq_linear_bwd", "tq_codes_transpose",
+                 "tq_linear_fwd_batched", "tq_device_status"):
         getattr(lib, name).restype = ctypes.c_int
     lib.tq_last_error.restype = ctypes.c_char_p
     lib.tq_last_error.argtypes = []
@@ -151,11 +153,23 @@ def linear_fwd(x: torch.Tensor, codes: torch.Tensor, scales: torch.Tensor, g: in
     return y
 
 
+def codes_transpose(codes: torch.Tensor, k: int, out: Optional[torch.Tensor] = None, stream=None):
+    """Packed codes of W^T (uint32 bit patterns in int32) ``[K, 4 * ceil(N / 64)]``."""
+    n = codes.shape[0]
+    if out is None:
+        out = torch.empty((k, 4 * ((n + 63) // 64)), dtype=torch.int32, device=codes.device)
+    _check(load().tq_codes_transpose(_ptr(codes), n, k, _ptr(out), _stream(stream)))
+    return out
+
+
 def linear_bwd(dy: torch.Tensor, x: Optional[torch.Tensor], codes: torch.Tensor,
                scales: torch.Tensor, k: int, g: int, want_dx: bool = True, want_dw: bool = True,
                dx_dtype=torch.float32, dx: Optional[torch.Tensor] = None,
-               dw: Optional[torch.Tensor] = None, accumulate_dw: bool = False, stream=None):
-    """STE backward; returns ``(dx [M, K] or None, dw fp32 [N, K] or None)``."""
+               dw: Optional[torch.Tensor] = None, accumulate_dw: bool = False,
+               codes_t: Optional[torch.Tensor] = None, stream=None):
+    """STE backward; returns ``(dx [M, K] or None, dw fp32 [N, K] or None)``.
+
+    ``codes_t`` (from ``codes_transpose``) selects the faster dX path."""
     m, n = dy.shape
     if want_dx and dx is None:
         dx = torch.empty((m, k), dtype=dx_dtype, device=dy.device)
@@ -165,7 +179,8 @@ def linear_bwd(dy: torch.Tensor, x: Optional[torch.Tensor], codes: torch.Tensor,
         dx = None
     if not want_dw:
         dw = None
-    _check(load().tq_linear_bwd(_ptr(dy), _ptr(x), m, n, k, _ptr(codes), _ptr(scales), g,
+    _check(load().tq_linear_bwd(_ptr(dy), _ptr(x), m, n, k, _ptr(codes), _ptr(codes_t),
+                                _ptr(scales), g,
                                 _ptr(dx), _out_code(dx.dtype) if dx is not None else OUT_F32,
                                 _ptr(dw), int(accumulate_dw), _stream(stream)))
     return dx, dw

@@ -96,15 +96,27 @@ def test_linear_fwd_rejects_before_launch(lib, args, status):
 
 
 @pytest.mark.parametrize("args,status", [
-    ((FAKE, FAKE, 4, 60, 256, FAKE, FAKE, 32, FAKE, 0, FAKE, 0, None), 2),  # n % 8
-    ((FAKE, FAKE, 4, 64, 256, FAKE, FAKE, 32, None, 0, None, 0, None), 1),  # no output
-    ((FAKE, None, 4, 64, 256, FAKE, FAKE, 32, None, 0, FAKE, 0, None), 1),  # dw needs x
-    ((None, FAKE, 4, 64, 256, FAKE, FAKE, 32, FAKE, 0, None, 0, None), 1),  # dx needs dy
-    ((FAKE, FAKE, 4, 64, 256, FAKE, FAKE, 32, FAKE, 3, None, 0, None), 1),  # bad dtype
-    ((FAKE, FAKE, 4, 64, 256, None, FAKE, 32, FAKE, 0, None, 0, None), 1),  # dx needs codes
+    ((FAKE, FAKE, 4, 60, 256, FAKE, None, FAKE, 32, FAKE, 0, FAKE, 0, None), 2),  # n % 8
+    ((FAKE, FAKE, 4, 64, 256, FAKE, None, FAKE, 32, None, 0, None, 0, None), 1),  # no output
+    ((FAKE, None, 4, 64, 256, FAKE, None, FAKE, 32, None, 0, FAKE, 0, None), 1),  # dw needs x
+    ((None, FAKE, 4, 64, 256, FAKE, None, FAKE, 32, FAKE, 0, None, 0, None), 1),  # dx needs dy
+    ((FAKE, FAKE, 4, 64, 256, FAKE, None, FAKE, 32, FAKE, 3, None, 0, None), 1),  # bad dtype
+    ((FAKE, FAKE, 4, 64, 256, None, None, FAKE, 32, FAKE, 0, None, 0, None), 1),  # dx needs codes
+    ((FAKE, FAKE, 4, 64, 256, None, MIS, FAKE, 32, FAKE, 0, None, 0, None), 1),   # misaligned codes_t
 ])
 def test_linear_bwd_rejects_before_launch(lib, args, status):
     assert lib.tq_linear_bwd(*args) == status
+
+
+@pytest.mark.parametrize("args,status", [
+    ((FAKE, 64, 200, FAKE, None), 1),   # k % 16
+    ((None, 64, 256, FAKE, None), 1),   # null codes
+    ((FAKE, 64, 256, MIS, None), 1),    # misaligned output
+    ((FAKE, -1, 256, FAKE, None), 1),   # negative
+    ((None, 0, 256, None, None), 0),    # empty
+])
+def test_codes_transpose_rejects_before_launch(lib, args, status):
+    assert lib.tq_codes_transpose(*args) == status
 
 
 def test_batched_rejects_before_launch(lib):

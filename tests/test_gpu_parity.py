@@ -132,10 +132,27 @@ def test_linear_parity(tq, n, k, m, g):
     xd, dyd = x.cuda(), dy.cuda()
     y = tq.linear_fwd(xd, codes, s, g)
     dx, dw = tq.linear_bwd(dyd, xd, codes, s, k, g)
+    ct = tq.codes_transpose(codes, k)
+    dxt, _ = tq.linear_bwd(dyd, xd, codes, s, k, g, want_dw=False, codes_t=ct)
     tq.device_status()
     check_close(y, O.linear_fwd(x, w_hat), "Y")
     check_close(dx, O.linear_bwd_dx(dy, w_hat), "dX")
+    check_close(dxt, O.linear_bwd_dx(dy, w_hat), "dX (codes_t)")
     check_close(dw, O.linear_bwd_dw(dy, x), "dW")
+
+
+@pytest.mark.parametrize("n,k", [(200, 192), (64, 64), (520, 1024), (1000, 2048), (8512, 2048)])
+def test_codes_transpose_layout(tq, n, k):
+    """tq_codes_transpose against the oracle's packing of the transposed codes."""
+    rs = np.random.default_rng(n + k)
+    c = rs.choice(np.array([-1, 0, 1], dtype=np.int8), size=(n, k))
+    codes = torch.from_numpy(O.pack(c).view(np.int32)).cuda()
+    ct = tq.codes_transpose(codes, k)
+    tq.device_status()
+    npad = 64 * ((n + 63) // 64)
+    cpad = np.zeros((k, npad), dtype=np.int8)
+    cpad[:, :n] = c.T
+    assert np.array_equal(codes_u32(ct), O.pack(cpad))
 
 
 def test_linear_bf16_outputs_are_rounded_fp32(tq):
@@ -241,7 +258,10 @@ def test_linear_mamba2_prefill_sampled(tq, proj):
     xd, dyd = x.cuda(), dy.cuda()
     y = tq.linear_fwd(xd, codes, s, g)
     dx, dw = tq.linear_bwd(dyd, xd, codes, s, k, g)
+    ct = tq.codes_transpose(codes, k)
+    dxt, _ = tq.linear_bwd(dyd, xd, codes, s, k, g, want_dw=False, codes_t=ct)
     tq.device_status()
+    assert torch.equal(dxt, dx)  # same operands, same MMA order
     rs = np.random.default_rng(1)
     rows = np.sort(rs.choice(m, 64, replace=False))
     nrows = np.sort(rs.choice(n, 64, replace=False))
