@@ -301,7 +301,8 @@ def decode_sweep(tq, m_list, steps, warmup):
 
 
 def quantize_sweep(tq, steps, warmup):
-    """tq_quantize over the 96 projections of 48 blocks (the per-step requantize)."""
+    """tq_quantize_batched over the 96 projections of 48 blocks in one launch (the
+    per-step requantize)."""
     gen = torch.Generator(device="cuda")
     gen.manual_seed(99)
     ws = [torch.randn(shape, generator=gen, device="cuda") * 0.02
@@ -311,9 +312,10 @@ def quantize_sweep(tq, steps, warmup):
              torch.empty((w.shape[0], w.shape[1] // G), dtype=torch.int32, device="cuda"))
             for w in ws]
 
+    arr = tq.quant_batch([(w, *o) for w, o in zip(ws, outs)])
+
     def run():
-        for w, o in zip(ws, outs):
-            tq.quantize(w, G, out=o)
+        tq.quantize_batched(arr, G)
 
     for _ in range(warmup):
         run()

@@ -84,6 +84,30 @@ TQ_API tq_status tq_quantize(const float* w, int64_t n, int64_t k, int32_t g,
                       uint32_t* codes, float* scales, int32_t* zero_counts,
                       void* stream);
 
+/* Largest entry count of the batched calls. */
+#define TQ_MAX_BATCH 256
+
+/* One matrix of a batched quantize call (tq_quantize_batched). */
+typedef struct {
+  const float* w;         /* fp32 [n][k] latent weights          */
+  uint32_t* codes;        /* out: uint32 [n][k/16]               */
+  float* scales;          /* out: fp32 [n][k/g]                  */
+  int32_t* zero_counts;   /* out: int32 [n][k/g]                 */
+  int64_t n;              /* rows                                */
+  int64_t k;              /* columns, k % 16 == 0 and k % g == 0 */
+} tq_quant_desc;
+
+/*
+ * tq_quantize_batched — tq_quantize of many matrices with the same group size
+ * in one launch (e.g. the per-step requantize of every in_proj and out_proj of a
+ * 48-block model, §3.1: the scale is recomputed at every forward). Each entry
+ * gets exactly tq_quantize's result. descs is a HOST array (copied into the
+ * launch; not kept); count <= TQ_MAX_BATCH; the outputs of different entries
+ * must not overlap.
+ */
+TQ_API tq_status tq_quantize_batched(const tq_quant_desc* descs, int32_t count, int32_t g,
+                                     void* stream);
+
 /*
  * tq_linear_fwd — W1.58A16 forward (§3.1, "W1.58A16" of the title):
  *   y[m][n] = sum_k x[m][k] * s[n][k/g] * code[n][k].
@@ -142,8 +166,6 @@ typedef struct {
   int32_t g;              /* group size                          */
   int32_t y_dtype;        /* tq_out_dtype                        */
 } tq_fwd_desc;
-
-#define TQ_MAX_BATCH 256
 
 /*
  * tq_linear_fwd_batched — the decode forward of many matrices in one launch

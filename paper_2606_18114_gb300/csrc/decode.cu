@@ -352,13 +352,11 @@ cudaError_t launch_decode(DecodeBatch& b, int num_sms, cudaStream_t stream) {
   const size_t smem = kSmemBytes + 128;
   cudaError_t e;
   if (b.m > 8) {
-    e = cudaFuncSetAttribute(decode_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(smem));
+    e = ensure_smem_limit<decode_kernel<true>>(static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     decode_kernel<true><<<static_cast<unsigned>(blocks), kThreads, smem, stream>>>(b);
   } else {
-    e = cudaFuncSetAttribute(decode_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(smem));
+    e = ensure_smem_limit<decode_kernel<false>>(static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     decode_kernel<false><<<static_cast<unsigned>(blocks), kThreads, smem, stream>>>(b);
   }

@@ -39,28 +39,6 @@ constexpr int kNumBars = 2 * kStages + 4;
 constexpr int kBytes = kBarOff + kNumBars * 8 + 8;
 constexpr uint32_t kTmemCols = 512;
 
-__device__ __forceinline__ uint64_t policy_evict_last() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-
-__device__ __forceinline__ uint64_t policy_evict_first() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-
-__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap* map,
-                                                 uint32_t bar, int32_t x, int32_t y,
-                                                 uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(policy)
-      : "memory");
-}
-
 __global__ void __launch_bounds__(kThreads, 1)
     dw_gemm_kernel(const __grid_constant__ CUtensorMap tmap_x,
                    const __grid_constant__ CUtensorMap tmap_dy, const DwArgs args) {
@@ -225,8 +203,7 @@ size_t dw_smem_bytes() { return kBytes + 1024; }
 cudaError_t launch_dw_gemm(const CUtensorMap& tmap_x, const CUtensorMap& tmap_dy,
                            const DwArgs& a, int num_sms, cudaStream_t stream) {
   const size_t smem = dw_smem_bytes();
-  cudaError_t e = cudaFuncSetAttribute(dw_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
+  cudaError_t e = ensure_smem_limit<dw_gemm_kernel>(static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   const int64_t tiles = ((a.k + kDwTileK - 1) / kDwTileK) * ((a.n + kDwTileN - 1) / kDwTileN);
   const int64_t grid = tiles < num_sms ? tiles : num_sms;

@@ -5,11 +5,52 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 namespace tq {
+
+// Raise a kernel's dynamic shared-memory limit once per device (the attribute
+// persists; setting it on every launch costs host time on the launch path).
+template <auto kKernel>
+cudaError_t ensure_smem_limit(int bytes) {
+  static std::atomic<uint64_t> done{0};  // bit d: set on device d (d < 64), per kernel
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = dev < 64 ? (uint64_t{1} << dev) : 0;
+  if (bit != 0 && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(kKernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess && bit != 0) done.fetch_or(bit, std::memory_order_release);
+  return e;
+}
 
 // quantize.cu ----------------------------------------------------------------
 cudaError_t launch_quantize(const float* w, int64_t n, int64_t k, int g, uint32_t* codes,
-                            float* scales, int32_t* zeros, int num_sms, cudaStream_t stream);
+                            float* scales, int32_t* zeros, int* status, int num_sms,
+                            cudaStream_t stream);
+
+// Many matrices (same group size) in one launch.
+struct QuantMat {
+  const float* w;   // fp32 [n][k], flat
+  uint32_t* codes;  // uint32 [n][k/16]
+  float* scales;    // fp32 [n][k/g]
+  int32_t* zeros;   // int32 [n][k/g]
+  int64_t total;    // n * k
+  int64_t stage0;   // first stage of this matrix (set by the launcher)
+};
+
+template <int kMax>
+struct QuantBatch {
+  QuantMat mats[kMax];
+  int64_t nstages;  // set by the launcher
+  int32_t count;
+  int32_t pad;
+};
+
+constexpr int kQuantMaxMats = 256;
+
+cudaError_t launch_quantize_batched(QuantBatch<kQuantMaxMats>& batch, int g, int* status,
+                                    int num_sms, cudaStream_t stream);
 
 // codes [n][k/16] -> codes_t [k][4 * ceil(n / 64)] (the codes of W^T).
 cudaError_t launch_transpose_codes(const uint32_t* codes, int64_t n, int64_t k, uint32_t* codes_t,

@@ -3,110 +3,297 @@
 //
 // The weight matrix is treated as one flat array: groups (g | k) and code words
 // (16 | k) never straddle a row, so group j of row n is flat group n*(k/g)+j and
-// the outputs are flat arrays too. Each lane owns 16 consecutive weights — one
-// code word — read as four 16-byte loads; a warp covers 512 weights per unit and
-// keeps two units of loads in flight. A group spans g/16 consecutive lanes and is
-// reduced with log2(g/16) xor-shuffles; the zero count of a word is
-// 16 - popc(word & 0x5555...) because every non-zero code has its low bit set.
+// the outputs are flat arrays too.
+//
+// Streaming: a persistent grid (two CTAs per SM) splits the flat array into
+// stages of 8192 weights (32 KB), claimed one at a time from a per-launch atomic
+// counter (SMs do not all receive HBM data at the same rate; static equal shares
+// left the slowest CTA ~40% behind). One producer thread keeps a ring of kStages
+// stages in flight with
+// cp.async.bulk (L2 evict-first: the latent weights are read once), so the
+// loads never wait for the arithmetic; sixteen consumer warps split every stage,
+// 512 weights each, and release the slot through an "empty" mbarrier. Two CTAs
+// per SM keep 32 blocks of 512 weights in process per SM, which the per-block
+// latency (shuffle chain, reductions) needs to keep pace with HBM.
+//
+// Consumer: each lane owns 16 consecutive weights — one code word. A group
+// spans g/16 consecutive lanes; its |w| sum is reduced with log2(g/16)
+// xor-shuffles and its zero count with one redux.sync over the group's lanes (the
+// zero count of a word is 16 - popc(word & 0x5555...) because every non-zero code
+// has its low bit set).
 //
 // Code decision. The code is +-1 iff fl32(|w| / s) > 0.5 (round half to even sends
 // 0.5 to 0; the clip maps everything beyond 1.5 to +-1). The fp32 quotient exceeds
 // 0.5 exactly when the real quotient exceeds the midpoint 0.5 + 2^-25 between 0.5
-// and its successor, i.e. when |w| - s/2 > s * 2^-25. For s >= 2^-100 both s/2
-// and s * 2^-25 are exact, and |w| - s/2 is exact whenever s/4 <= |w| <= s
-// (Sterbenz); outside that band its rounded value still has the right side of
-// the threshold. So one fused multiply-add and one compare reproduce the
-// correctly rounded division bit for bit. Smaller scales take the division.
+// and its successor, i.e. when |w| > s (1/2 + 2^-25). For a normal s that
+// threshold lies strictly between s/2 and the next fp32 value above s/2, so on
+// fp32 inputs the test is |w| > s/2 — one comparison reproduces the correctly
+// rounded division bit for bit (s/2 is exact for s >= 2^-125). Scales below
+// 2^-100 take the division.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
 #include "kernels.cuh"
+#include "ptx.cuh"
 
 namespace tq {
 namespace {
 
-constexpr int kUnit = 512;    // weights per warp per unit
-constexpr int kUnroll = 2;    // units per warp iteration (loads in flight)
-constexpr int kThreads = 256;
+constexpr int kUnit = 512;                      // weights per consumer warp per stage
+constexpr int kConsumers = 16;                  // consumer warps
+constexpr int kThreads = (kConsumers + 1) * 32; // + one producer warp
+constexpr int kStageW = kConsumers * kUnit;     // 8192 weights per stage
+constexpr int kStageBytes = kStageW * 4;        // 32 KB
+constexpr int kStages = 3;                      // per CTA; two CTAs per SM
+constexpr int kCtasPerSm = 2;
+constexpr int kSmemBytes = kStages * kStageBytes + 2 * kStages * 8 + 128;
 
-__device__ __forceinline__ uint32_t code_bits(float w, float s, float t, bool tiny_s) {
-  const bool nz = tiny_s ? fabsf(__fdiv_rn(w, s)) > 0.5f : __fmaf_rn(-0.5f, s, fabsf(w)) > t;
-  const uint32_t neg = __float_as_uint(w) >> 31;
-  return nz ? (1u | (neg << 1)) : 0u;
+// w |= bit when a > h (one compare and one predicated OR).
+__device__ __forceinline__ void or_if_gt(uint32_t& w, float a, float h, uint32_t bit) {
+  asm("{\n\t.reg .pred p;\n\tsetp.gt.f32 p, %1, %2;\n\t@p or.b32 %0, %0, %3;\n\t}"
+      : "+r"(w)
+      : "f"(a), "f"(h), "r"(bit));
 }
 
-template <int G>
-__global__ void __launch_bounds__(kThreads) quantize_kernel(const float* __restrict__ w,
-                                                            int64_t total,
-                                                            uint32_t* __restrict__ codes,
-                                                            float* __restrict__ scales,
-                                                            int32_t* __restrict__ zeros) {
+// Code word of 16 consecutive weights; code j at bit p_j = 16*(j&1) + 2*(j>>1),
+// high bit the sign, low bit "non-zero".
+//   nz:  bit p_j set iff |w_j| > s/2 (fast path) or fl(|w_j| / s) > 0.5.
+//   neg: bit p_j + 1 set iff w_j < 0 (sign bit), for every j. The sign bits of
+//        weights 2i and 2i+1 (bound for bits 2i+1 and 2i+17) are gathered by one
+//        byte permute (bits 15 and 31), one shift and one masked OR.
+//   word = nz | (neg & (nz << 1)): the sign only where the code is non-zero.
+template <bool kDivide>
+__device__ __forceinline__ uint32_t code_word(const float (&x)[16], float s) {
+  uint32_t nz = 0, neg = 0;
+  if (kDivide) {
+#pragma unroll
+    for (int j = 0; j < 16; ++j)
+      or_if_gt(nz, fabsf(__fdiv_rn(x[j], s)), 0.5f, 1u << (16 * (j & 1) + 2 * (j >> 1)));
+  } else {
+    const float h = 0.5f * s;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) or_if_gt(nz, fabsf(x[j]), h, 1u << (16 * (j & 1) + 2 * (j >> 1)));
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const uint32_t hi = __byte_perm(__float_as_uint(x[2 * i]), __float_as_uint(x[2 * i + 1]), 0x7632);
+    neg |= (hi >> (14 - 2 * i)) & ((1u << (2 * i + 1)) | (1u << (2 * i + 17)));
+  }
+  return nz | (neg & (nz << 1));
+}
+
+// Stage scheduler of one launch: {next dynamic stage, CTAs done}. Zero at the
+// start of a launch; the last CTA to finish claiming puts both back to zero.
+// Launches take the slots in turn, so up to kSchedSlots launches may be in
+// flight at once.
+constexpr int kSchedSlots = 256;
+__device__ uint32_t g_sched[kSchedSlots][2];
+
+// Matrix d of a batch owns the global stages [stage0, stage0 + ceil(total / kStageW));
+// a stage never spans two matrices (a matrix's last stage may be short).
+__device__ __forceinline__ int find_stage_mat(const QuantMat* mats, int count, int64_t st) {
+  int lo = 0, hi = count - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (mats[mid].stage0 <= st) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+template <int G, int kMax>
+__global__ void __launch_bounds__(kThreads, kCtasPerSm)
+    quantize_kernel(const __grid_constant__ QuantBatch<kMax> b, uint32_t* sched, int* status) {
   static_assert(G == 32 || G == 64 || G == 128 || G == 256 || G == 512, "group size");
+  static_assert(kStageW % G == 0, "a group never straddles a stage");
   constexpr int kLanesPerGroup = G / 16;
   constexpr float kInvG = 1.0f / G;  // exact: G is a power of two
-  const int lane = threadIdx.x & 31;
-  const int64_t warp0 = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
-  const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * kThreads) >> 5;
-  const int64_t nunits = (total + kUnit - 1) / kUnit;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ int64_t stage_of[kStages];  // local stage held by each slot; -1: end of stream
+  __shared__ int mat_of[kStages];        // its matrix
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) &
+                                             ~static_cast<uintptr_t>(127));
+  const uint32_t ring = smem_u32(smem);
+  const uint32_t bars = ring + kStages * kStageBytes;
+  auto full_bar = [&](int s) { return bars + 8 * s; };
+  auto empty_bar = [&](int s) { return bars + 8 * (kStages + s); };
 
-  for (int64_t u0 = warp0 * kUnroll; u0 < nunits; u0 += nwarps * kUnroll) {
-    float4 v[kUnroll][4];
-#pragma unroll
-    for (int r = 0; r < kUnroll; ++r) {
-      const int64_t e = (u0 + r) * kUnit + lane * 16;
-      const bool in = e < total;
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        v[r][j] = in ? __ldg(reinterpret_cast<const float4*>(w + e) + j)
-                     : make_float4(0.f, 0.f, 0.f, 0.f);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int64_t nstages = b.nstages;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), kConsumers);
     }
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  if (warp == kConsumers) {
+    // ------------------------------------------------------------ producer
+    // The first ring's worth of stages is dealt round-robin (no claim latency
+    // before the first loads); later stages are claimed one at a time from the
+    // launch's counter, so SMs that receive their data faster take more of them
+    // and all CTAs end together.
+    if (lane == 0) {
+      const uint64_t policy = policy_evict_first();
+      const int64_t dealt = static_cast<int64_t>(kStages) * gridDim.x;
+      int round0 = 0;
+      auto claim = [&]() -> int64_t {
+        if (round0 < kStages) return blockIdx.x + static_cast<int64_t>(round0++) * gridDim.x;
+        return dealt + atomicAdd(&sched[0], 1u);
+      };
+      int slot = 0;
+      uint32_t parity = 0;  // phase parity of the slot's current round
+      int64_t issued = 0;
+      bool ok = true;
+      int64_t st = claim();
+      for (;;) {
+        if (issued >= kStages && !mbar_wait(empty_bar(slot), parity ^ 1u, status)) {
+          ok = false;
+          break;
+        }
+        if (st >= nstages) {  // end of the stream: an empty stage tells the consumers
+          stage_of[slot] = -1;
+          mbar_arrive(full_bar(slot));
+          break;
+        }
+        const int d = kMax == 1 ? 0 : find_stage_mat(b.mats, b.count, st);
+        const QuantMat& mt = b.mats[d];
+        const int64_t ls = st - mt.stage0;
+        const int64_t e0 = ls * kStageW;
+        const int64_t cnt = mt.total - e0 < kStageW ? mt.total - e0 : kStageW;
+        const uint32_t bytes = static_cast<uint32_t>(cnt) * 4u;
+        stage_of[slot] = ls;
+        mat_of[slot] = d;
+        mbar_arrive_expect_tx(full_bar(slot), bytes);
+        bulk_load(ring + slot * kStageBytes, mt.w + e0, bytes, full_bar(slot), policy);
+        st = claim();  // a counter claim is in flight during the wait above
+        ++issued;
+        if (++slot == kStages) {
+          slot = 0;
+          parity ^= 1u;
+        }
+      }
+      // this CTA claims no more: the last CTA to get here resets the scheduler
+      __threadfence();
+      if (atomicAdd(&sched[1], 1u) == gridDim.x - 1) {
+        atomicExch(&sched[0], 0u);
+        atomicExch(&sched[1], 0u);
+      }
+      // Nothing may still write this CTA's ring when it exits. Normally the
+      // consumers have waited for every stage before they see the end marker;
+      // if they gave up, wait here for the stages issued last (a slot's newest
+      // phase is its last load: no end marker was written on this path).
+      if (!ok) {
+        for (int64_t j = issued > kStages ? issued - kStages : 0; j < issued; ++j) {
+          if (!mbar_wait(full_bar(static_cast<int>(j % kStages)),
+                         static_cast<uint32_t>((j / kStages) & 1), status))
+            break;
+        }
+      }
+    }
+    return;
+  }
+
+  // -------------------------------------------------------------- consumers
+  int slot = 0;
+  uint32_t parity = 0;
+  for (;;) {
+    if (!warp_wait(full_bar(slot), parity, status)) return;
+    const int64_t ls = stage_of[slot];
+    if (ls < 0) return;
+    const QuantMat& mt = b.mats[kMax == 1 ? 0 : mat_of[slot]];
+    const int64_t total = mt.total;
+    const int64_t base = ls * kStageW + warp * kUnit;
+    const int64_t e = base + lane * 16;
+    if (e < total) {
+      // lanes of this block that hold weights; a multiple of g/16 (g | total)
+      const int64_t rem = total - base;
+      const unsigned live = rem >= kUnit ? 0xffffffffu : (1u << (rem >> 4)) - 1u;
+      const float4* src = reinterpret_cast<const float4*>(smem + slot * kStageBytes +
+                                                          (warp * kUnit + lane * 16) * 4);
+      float4 v[4];
 #pragma unroll
-    for (int r = 0; r < kUnroll; ++r) {
-      const int64_t e = (u0 + r) * kUnit + lane * 16;
+      for (int j = 0; j < 4; ++j) v[j] = src[j];
       float sum = 0.f;
 #pragma unroll
       for (int j = 0; j < 4; ++j)
-        sum += (fabsf(v[r][j].x) + fabsf(v[r][j].y)) + (fabsf(v[r][j].z) + fabsf(v[r][j].w));
+        sum += (fabsf(v[j].x) + fabsf(v[j].y)) + (fabsf(v[j].z) + fabsf(v[j].w));
 #pragma unroll
-      for (int off = 1; off < kLanesPerGroup; off <<= 1)
-        sum += __shfl_xor_sync(0xffffffffu, sum, off);
-      const float s = sum * kInvG;            // s = (1/g) * sum |w|
-      const float t = s * 0x1p-25f;           // half an ulp of 0.5, in units of s
+      for (int off = 1; off < kLanesPerGroup; off <<= 1) sum += __shfl_xor_sync(live, sum, off);
+      const float s = sum * kInvG;  // s = (1/g) * sum |w|
+      const float x[16] = {v[0].x, v[0].y, v[0].z, v[0].w, v[1].x, v[1].y, v[1].z, v[1].w,
+                           v[2].x, v[2].y, v[2].z, v[2].w, v[3].x, v[3].y, v[3].z, v[3].w};
+      // scales below 2^-100 (all-zero or denormal groups) take the division
       const bool tiny = s < 0x1p-100f;
-      const float x[16] = {v[r][0].x, v[r][0].y, v[r][0].z, v[r][0].w,
-                           v[r][1].x, v[r][1].y, v[r][1].z, v[r][1].w,
-                           v[r][2].x, v[r][2].y, v[r][2].z, v[r][2].w,
-                           v[r][3].x, v[r][3].y, v[r][3].z, v[r][3].w};
-      uint32_t word = 0;
-#pragma unroll
-      for (int i = 0; i < 16; ++i)  // code i at bit 16*(i&1) + 2*(i>>1)
-        word |= code_bits(x[i], s, t, tiny) << (16 * (i & 1) + 2 * (i >> 1));
-      int zc = 16 - __popc(word & 0x55555555u);
-#pragma unroll
-      for (int off = 1; off < kLanesPerGroup; off <<= 1) zc += __shfl_xor_sync(0xffffffffu, zc, off);
-      if (e < total) {
-        codes[e >> 4] = word;
-        if ((lane & (kLanesPerGroup - 1)) == 0) {
-          scales[e / G] = s;
-          zeros[e / G] = zc;
-        }
+      const uint32_t word = __any_sync(live, tiny)
+                                ? (tiny ? code_word<true>(x, s) : code_word<false>(x, s))
+                                : code_word<false>(x, s);
+      const unsigned gmask =
+          kLanesPerGroup == 32 ? 0xffffffffu
+                               : ((1u << kLanesPerGroup) - 1u) << (lane & ~(kLanesPerGroup - 1));
+      const int zc = static_cast<int>(
+          __reduce_add_sync(gmask, static_cast<unsigned>(16 - __popc(word & 0x55555555u))));
+      mt.codes[e >> 4] = word;
+      if ((lane & (kLanesPerGroup - 1)) == 0) {
+        mt.scales[e / G] = s;
+        mt.zeros[e / G] = zc;
       }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(empty_bar(slot));
+    if (++slot == kStages) {
+      slot = 0;
+      parity ^= 1u;
     }
   }
 }
 
-template <int G>
-cudaError_t launch(const float* w, int64_t total, uint32_t* codes, float* scales, int32_t* zeros,
-                   int num_sms, cudaStream_t stream) {
-  const int64_t nunits = (total + kUnit - 1) / kUnit;
-  const int64_t warps_needed = (nunits + kUnroll - 1) / kUnroll;
-  const int64_t warps_per_block = kThreads / 32;
-  int64_t blocks = (warps_needed + warps_per_block - 1) / warps_per_block;
-  const int64_t cap = static_cast<int64_t>(num_sms) * 8;  // 8 resident blocks per SM
-  if (blocks > cap) blocks = cap;
-  quantize_kernel<G><<<static_cast<unsigned>(blocks), kThreads, 0, stream>>>(w, total, codes,
-                                                                           scales, zeros);
+// Device address of g_sched, looked up once per device.
+uint32_t* sched_base() {
+  static std::atomic<uintptr_t> base[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+  if (dev < 64) {
+    const uintptr_t p = base[dev].load(std::memory_order_acquire);
+    if (p != 0) return reinterpret_cast<uint32_t*>(p);
+  }
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_sched) != cudaSuccess) return nullptr;
+  if (dev < 64) base[dev].store(reinterpret_cast<uintptr_t>(p), std::memory_order_release);
+  return static_cast<uint32_t*>(p);
+}
+
+template <int G, int kMax>
+cudaError_t launch(const QuantBatch<kMax>& b, int* status, int num_sms, cudaStream_t stream) {
+  static std::atomic<uint32_t> seq{0};
+  if (b.nstages <= 0) return cudaSuccess;
+  if (b.nstages >= (int64_t{1} << 31)) return cudaErrorInvalidValue;
+  const int64_t cap = static_cast<int64_t>(num_sms) * kCtasPerSm;
+  const int64_t blocks = b.nstages < cap ? b.nstages : cap;
+  cudaError_t e = ensure_smem_limit<quantize_kernel<G, kMax>>(kSmemBytes);
+  if (e != cudaSuccess) return e;
+  uint32_t* sched = sched_base();
+  if (sched == nullptr) return cudaErrorInvalidSymbol;
+  sched += 2 * (seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
+  quantize_kernel<G, kMax><<<static_cast<unsigned>(blocks), kThreads, kSmemBytes, stream>>>(
+      b, sched, status);
   return cudaGetLastError();
+}
+
+template <int kMax>
+cudaError_t launch_g(const QuantBatch<kMax>& b, int g, int* status, int num_sms,
+                     cudaStream_t stream) {
+  switch (g) {
+    case 32: return launch<32, kMax>(b, status, num_sms, stream);
+    case 64: return launch<64, kMax>(b, status, num_sms, stream);
+    case 128: return launch<128, kMax>(b, status, num_sms, stream);
+    case 256: return launch<256, kMax>(b, status, num_sms, stream);
+    case 512: return launch<512, kMax>(b, status, num_sms, stream);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 // codes [n][k/16] -> codes_t [k][ldt]: a 128 x 128 (n x k) tile per block. The tile's
@@ -155,16 +342,24 @@ cudaError_t launch_transpose_codes(const uint32_t* codes, int64_t n, int64_t k, 
 }
 
 cudaError_t launch_quantize(const float* w, int64_t n, int64_t k, int g, uint32_t* codes,
-                            float* scales, int32_t* zeros, int num_sms, cudaStream_t stream) {
-  const int64_t total = n * k;
-  switch (g) {
-    case 32: return launch<32>(w, total, codes, scales, zeros, num_sms, stream);
-    case 64: return launch<64>(w, total, codes, scales, zeros, num_sms, stream);
-    case 128: return launch<128>(w, total, codes, scales, zeros, num_sms, stream);
-    case 256: return launch<256>(w, total, codes, scales, zeros, num_sms, stream);
-    case 512: return launch<512>(w, total, codes, scales, zeros, num_sms, stream);
-    default: return cudaErrorInvalidValue;
+                            float* scales, int32_t* zeros, int* status, int num_sms,
+                            cudaStream_t stream) {
+  QuantBatch<1> b{};
+  b.mats[0] = QuantMat{w, codes, scales, zeros, n * k, 0};
+  b.count = 1;
+  b.nstages = (n * k + kStageW - 1) / kStageW;
+  return launch_g<1>(b, g, status, num_sms, stream);
+}
+
+cudaError_t launch_quantize_batched(QuantBatch<kQuantMaxMats>& b, int g, int* status,
+                                    int num_sms, cudaStream_t stream) {
+  int64_t st = 0;
+  for (int d = 0; d < b.count; ++d) {
+    b.mats[d].stage0 = st;
+    st += (b.mats[d].total + kStageW - 1) / kStageW;
   }
+  b.nstages = st;
+  return launch_g<kQuantMaxMats>(b, g, status, num_sms, stream);
 }
 
 }  // namespace tq

@@ -184,6 +184,7 @@ tq_status fwd_checked(const void* x, int64_t m, int64_t k, const uint32_t* codes
 }
 
 static_assert(tq::kDecodeMaxMats >= TQ_MAX_BATCH, "decode batch table");
+static_assert(tq::kQuantMaxMats >= TQ_MAX_BATCH, "quantize batch table");
 
 // Forward for m <= 16 tokens: the HBM-streaming decode kernel over all matrices.
 tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
@@ -247,9 +248,8 @@ TQ_API const char* tq_last_error(void) { return g_err; }
 
 TQ_API const char* tq_version(void) { return "tq 0.1 (sm_103a)"; }
 
-TQ_API tq_status tq_quantize(const float* w, int64_t n, int64_t k, int32_t g, uint32_t* codes,
-                             float* scales, int32_t* zero_counts, void* stream) {
-  g_err[0] = 0;
+tq_status check_quantize_args(const float* w, int64_t n, int64_t k, int32_t g, const uint32_t* codes,
+                               const float* scales, const int32_t* zero_counts) {
   if (n < 0 || k < 0) return fail(TQ_ERR_INVALID_ARG, "negative size");
   if (log2_group(g) < 0) return fail(TQ_ERR_INVALID_ARG, "group size %d not in {32..512}", g);
   if (k % 16 != 0) return fail(TQ_ERR_INVALID_ARG, "k=%lld is not a multiple of 16", (long long)k);
@@ -260,10 +260,46 @@ TQ_API tq_status tq_quantize(const float* w, int64_t n, int64_t k, int32_t g, ui
   TQ_TRY(check_ptr(codes, "codes"));
   TQ_TRY(check_ptr(scales, "scales"));
   TQ_TRY(check_ptr(zero_counts, "zero_counts"));
+  return TQ_OK;
+}
+
+TQ_API tq_status tq_quantize(const float* w, int64_t n, int64_t k, int32_t g, uint32_t* codes,
+                             float* scales, int32_t* zero_counts, void* stream) {
+  g_err[0] = 0;
+  TQ_TRY(check_quantize_args(w, n, k, g, codes, scales, zero_counts));
+  if (n == 0 || k == 0) return TQ_OK;
   const DeviceInfo* dev = nullptr;
   TQ_TRY(device_info(&dev));
-  cudaError_t e = tq::launch_quantize(w, n, k, g, codes, scales, zero_counts, dev->num_sms,
-                                      static_cast<cudaStream_t>(stream));
+  cudaError_t e = tq::launch_quantize(w, n, k, g, codes, scales, zero_counts, dev->status,
+                                      dev->num_sms, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "quantize launch");
+}
+
+TQ_API tq_status tq_quantize_batched(const tq_quant_desc* descs, int32_t count, int32_t g,
+                                     void* stream) {
+  g_err[0] = 0;
+  if (count < 0 || count > TQ_MAX_BATCH)
+    return fail(TQ_ERR_INVALID_ARG, "count %d not in [0, %d]", count, TQ_MAX_BATCH);
+  if (count > 0 && descs == nullptr) return fail(TQ_ERR_INVALID_ARG, "descs is NULL");
+  if (log2_group(g) < 0) return fail(TQ_ERR_INVALID_ARG, "group size %d not in {32..512}", g);
+  thread_local tq::QuantBatch<tq::kQuantMaxMats> b;
+  b.count = 0;
+  for (int32_t i = 0; i < count; ++i) {
+    const tq_quant_desc& d = descs[i];
+    const tq_status st = check_quantize_args(d.w, d.n, d.k, g, d.codes, d.scales, d.zero_counts);
+    if (st != TQ_OK) {
+      char msg[sizeof(g_err)];
+      snprintf(msg, sizeof(msg), "%s", g_err);
+      return fail(st, "descs[%d]: %s", i, msg);
+    }
+    if (d.n == 0 || d.k == 0) continue;
+    b.mats[b.count++] = tq::QuantMat{d.w, d.codes, d.scales, d.zero_counts, d.n * d.k, 0};
+  }
+  if (b.count == 0) return TQ_OK;
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaError_t e = tq::launch_quantize_batched(b, g, dev->status, dev->num_sms,
+                                              static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? TQ_OK : cuda_fail(e, "quantize launch");
 }
 

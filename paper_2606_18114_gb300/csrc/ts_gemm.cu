@@ -452,8 +452,7 @@ cudaError_t launch_impl(const CUtensorMap& tb, const CUtensorMap& tc, const TsAr
   size_t smem = L::kBytes + 1024;
   if (smem < 116 * 1024) smem = 116 * 1024;
   auto kern = ts_gemm_kernel<MODE, BN>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
+  cudaError_t e = ensure_smem_limit<ts_gemm_kernel<MODE, BN>>(static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   const int64_t rows = MODE == kTsFwd ? a.wn : a.wk;
   const int64_t tiles = ((rows + 127) / 128) * ((a.m + BN - 1) / BN);

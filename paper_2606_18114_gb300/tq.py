@@ -16,6 +16,8 @@ __all__ = [
     "TqError",
     "load",
     "quantize",
+    "quantize_batched",
+    "quant_batch",
     "linear_fwd",
     "linear_bwd",
     "codes_transpose",
@@ -33,8 +35,9 @@ OUT_BF16 = 1
 STATUS = {0: "TQ_OK", 1: "TQ_ERR_INVALID_ARG", 2: "TQ_ERR_UNSUPPORTED", 3: "TQ_ERR_CUDA",
           4: "TQ_ERR_TIMEOUT"}
 # Every symbol include/tq.h declares.
-EXPORTS = ("tq_quantize", "tq_linear_fwd", "tq_linear_bwd", "tq_codes_transpose",
-           "tq_linear_fwd_batched", "tq_device_status", "tq_last_error", "tq_version")
+EXPORTS = ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
+           "tq_codes_transpose", "tq_linear_fwd_batched", "tq_device_status", "tq_last_error",
+           "tq_version")
 
 _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtq.so")
 _lib = None
@@ -44,6 +47,17 @@ class TqError(RuntimeError):
     def __init__(self, status: int, message: str):
         super().__init__(f"{STATUS.get(status, status)}: {message}")
         self.status = status
+
+
+class QuantDesc(ctypes.Structure):
+    _fields_ = [
+        ("w", ctypes.c_void_p),
+        ("codes", ctypes.c_void_p),
+        ("scales", ctypes.c_void_p),
+        ("zero_counts", ctypes.c_void_p),
+        ("n", ctypes.c_int64),
+        ("k", ctypes.c_int64),
+    ]
 
 
 class FwdDesc(ctypes.Structure):
@@ -70,13 +84,14 @@ def load(path: Optional[str] = None):
     lib = ctypes.CDLL(p)
     i64, i32, vp = ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p
     lib.tq_quantize.argtypes = [vp, i64, i64, i32, vp, vp, vp, vp]
+    lib.tq_quantize_batched.argtypes = [ctypes.POINTER(QuantDesc), i32, i32, vp]
     lib.tq_linear_fwd.argtypes = [vp, i64, i64, vp, vp, i64, i32, vp, i32, vp]
     lib.tq_linear_bwd.argtypes = [vp, vp, i64, i64, i64, vp, vp, vp, i32, vp, i32, vp, i32, vp]
     lib.tq_codes_transpose.argtypes = [vp, i64, i64, vp, vp]
     lib.tq_linear_fwd_batched.argtypes = [ctypes.POINTER(FwdDesc), i32, i64, vp]
     lib.tq_device_status.argtypes = [vp]
-    for name in ("tq_quantize", "tq_linear_fwd", "tq_linear_bwd", "tq_codes_transpose",
-                 "tq_linear_fwd_batched", "tq_device_status"):
+    for name in ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
+                 "tq_codes_transpose", "tq_linear_fwd_batched", "tq_device_status"):
         getattr(lib, name).restype = ctypes.c_int
     lib.tq_last_error.restype = ctypes.c_char_p
     lib.tq_last_error.argtypes = []
@@ -131,6 +146,26 @@ def quantize(w: torch.Tensor, g: int, out=None, stream=None):
     _check(load().tq_quantize(_ptr(w), n, k, g, _ptr(codes), _ptr(scales), _ptr(zeros),
                               _stream(stream)))
     return codes, scales, zeros
+
+
+def quant_batch(items: Sequence[tuple]):
+    """Descriptor array for ``quantize_batched`` (build once, call many times).
+
+    ``items``: tuples ``(w, codes, scales, zero_counts)`` of allocated tensors
+    (outputs written in place). The tensors must outlive the array's use.
+    """
+    arr = (QuantDesc * len(items))()
+    for i, (w, codes, scales, zeros) in enumerate(items):
+        arr[i] = QuantDesc(_ptr(w), _ptr(codes), _ptr(scales), _ptr(zeros), w.shape[0],
+                           w.shape[1])
+    return arr
+
+
+def quantize_batched(items, g: int, stream=None) -> None:
+    """``quantize`` of many fp32 matrices with one group size in one launch
+    (``items`` as for ``quant_batch``, or an array that it returned)."""
+    arr = items if isinstance(items, ctypes.Array) else quant_batch(items)
+    _check(load().tq_quantize_batched(arr, len(arr), g, _stream(stream)))
 
 
 def _out_code(dtype) -> int:

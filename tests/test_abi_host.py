@@ -129,3 +129,21 @@ def test_batched_rejects_before_launch(lib):
     assert lib.tq_linear_fwd_batched(arr, 1, 17, None) == 1   # m > 16
     assert lib.tq_linear_fwd_batched(arr, 300, 1, None) == 1  # count > max
     assert lib.tq_linear_fwd_batched(None, 0, 1, None) == 0   # nothing to do
+
+
+def test_quantize_batched_rejects_before_launch(lib):
+    from paper_2606_18114_gb300.tq import QuantDesc
+    arr = (QuantDesc * 3)()
+    arr[0] = QuantDesc(FAKE, FAKE, FAKE, FAKE, 8, 256)
+    arr[1] = QuantDesc(FAKE, FAKE, FAKE, FAKE, 8, 96)    # k % g (g = 64)
+    arr[2] = QuantDesc(MIS, FAKE, FAKE, FAKE, 8, 256)    # misaligned w
+    assert lib.tq_quantize_batched(arr, 2, 64, None) == 1
+    assert b"descs[1]" in lib.tq_last_error()
+    arr[1] = QuantDesc(None, None, None, None, 0, 256)   # empty entry: skipped
+    assert lib.tq_quantize_batched(arr, 3, 64, None) == 1
+    assert b"descs[2]" in lib.tq_last_error()
+    assert lib.tq_quantize_batched(arr, 1, 48, None) == 1     # bad group size
+    assert lib.tq_quantize_batched(arr, 300, 64, None) == 1   # count > max
+    assert lib.tq_quantize_batched(arr, -1, 64, None) == 1    # negative count
+    assert lib.tq_quantize_batched(None, 2, 64, None) == 1    # null descs
+    assert lib.tq_quantize_batched(None, 0, 64, None) == 0    # nothing to do

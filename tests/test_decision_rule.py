@@ -1,18 +1,19 @@
-"""The quantize kernel decides a code with a fused multiply-add instead of a
-division: code != 0 iff |w| - s/2 > s * 2^-25 (for s >= 2^-100). This checks,
-on the CPU in numpy fp32, that the rule agrees bit for bit with the correctly
-rounded fp32 quotient |w| / s > 0.5 that §3.1's round(clip(w/s)) implies —
-on random pairs and on pairs placed on every fp32 value around the tie."""
+"""The quantize kernel decides a code with one comparison instead of a division:
+code != 0 iff |w| > s/2 (for s >= 2^-100). The correctly rounded fp32 quotient
+|w| / s exceeds 0.5 exactly when the real quotient exceeds the midpoint
+0.5 + 2^-25 (the tie goes to the even 0.5), i.e. when |w| > s (1/2 + 2^-25); for
+a normal s that threshold lies strictly between s/2 and the next fp32 value
+above it, so the two conditions agree on every fp32 |w|. This checks, on the CPU
+in numpy fp32, that the rule agrees bit for bit with the quotient test that
+§3.1's round(clip(w/s)) implies — on random pairs, on every fp32 value around
+the tie, and on every 16-bit-prefix mantissa of s."""
 import numpy as np
 
 
 def rule(w, s):
     w = w.astype(np.float32)
     s = s.astype(np.float32)
-    # fma(-0.5, s, |w|): 0.5*s is exact; the difference rounded once to fp32
-    d = (np.abs(w).astype(np.float64) - 0.5 * s.astype(np.float64)).astype(np.float32)
-    t = (s * np.float32(2.0 ** -25)).astype(np.float32)
-    return d > t
+    return np.abs(w) > s * np.float32(0.5)  # 0.5 * s is exact for s >= 2^-125
 
 
 def division(w, s):
@@ -54,3 +55,15 @@ def test_rule_extremes():
     for w in (np.zeros(4, np.float32), s * np.float32(0.25), s, s * np.float32(4)):
         w = w.astype(np.float32)
         assert np.array_equal(rule(w, s), division(w, s))
+
+
+def test_rule_every_scale_mantissa():
+    # every s = (1 + i / 2^16) * 2^e, with w on the four fp32 values nearest s/2
+    i = np.arange(1 << 16, dtype=np.float64)
+    for e in (-100, -7, 0, 20):
+        s = ((1.0 + i / 65536.0) * 2.0 ** e).astype(np.float32)
+        half = (s * np.float32(0.5)).astype(np.float32)
+        up = np.nextafter(half, np.float32(np.inf))
+        down = np.nextafter(half, np.float32(0))
+        for w in (half, up, down, np.nextafter(up, np.float32(np.inf))):
+            assert np.array_equal(rule(w, s), division(w, s))

@@ -105,6 +105,61 @@ def test_quantize_mamba2_full(tq, proj, dist):
     assert (0.30 < ratio < 0.32) if dist == "gauss" else (0.36 < ratio < 0.39)
 
 
+def _quant_batched(tq, ws, g):
+    items = []
+    for w_np in ws:
+        w = torch.from_numpy(w_np).cuda()
+        n, k = w.shape
+        items.append((w, torch.empty((n, k // 16), dtype=torch.int32, device="cuda"),
+                      torch.empty((n, k // g), device="cuda"),
+                      torch.empty((n, k // g), dtype=torch.int32, device="cuda")))
+    tq.quantize_batched(items, g)
+    tq.device_status()
+    return items
+
+
+@pytest.mark.parametrize("g", [32, 128, 512])
+def test_quantize_batched_mixed(tq, g):
+    # shapes whose flat sizes end mid-stage, a one-group matrix and an empty one
+    shapes = [(7, 1024), (1, g), (300, 512), (0, 1024), (33, 4096), (2, 8192)]
+    ws = [synth.latent_weights(n, k, seed=i, dist="t3" if i % 2 else "gauss")
+          for i, (n, k) in enumerate(shapes)]
+    for w, (_, codes, s, z) in zip(ws, _quant_batched(tq, ws, g)):
+        if w.size:
+            check_quantize(w, g, codes, s, z)
+
+
+def test_quantize_batched_matches_single(tq):
+    ws = [synth.latent_weights(n, k, seed=40 + i) for i, (n, k) in
+          enumerate([(512, 2048), (64, 4096), (96, 256)] * 3)]
+    for w, (wt, codes, s, z) in zip(ws, _quant_batched(tq, ws, 64)):
+        c1, s1, z1 = tq.quantize(wt, 64)
+        tq.device_status()
+        assert torch.equal(codes, c1) and torch.equal(s, s1) and torch.equal(z, z1)
+
+
+def test_quantize_batched_48_layers_sampled(tq):
+    # every in_proj and out_proj of the 48 blocks (5 GB of latent weights, drawn
+    # on the device) in one launch; 8 rows of each matrix checked
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(1234)
+    items = []
+    for _ in range(48):
+        for p in ("in_proj", "out_proj"):
+            n, k = synth.MAMBA2_1P3B[p]
+            w = torch.randn((n, k), generator=gen, device="cuda") * 0.02
+            items.append((w, torch.empty((n, k // 16), dtype=torch.int32, device="cuda"),
+                          torch.empty((n, k // 128), device="cuda"),
+                          torch.empty((n, k // 128), dtype=torch.int32, device="cuda")))
+    tq.quantize_batched(items, 128)
+    tq.device_status()
+    rs = np.random.default_rng(5)
+    for w, codes, s, z in items:
+        rows = torch.from_numpy(np.sort(rs.choice(w.shape[0], 8, replace=False))).cuda()
+        check_quantize(to_np(w[rows]), 128, codes[rows], s[rows], z[rows])
+    del items
+
+
 # ------------------------------------------------------------------ linear
 def _setup(tq, n, k, m, g, seed=0, dy_std=1.0, dist="gauss"):
     w = synth.latent_weights(n, k, seed=seed, dist=dist)
