@@ -3,46 +3,100 @@
 // the layer is bound by weight traffic; 2-bit codes + fp32 group scales are 0.28
 // bytes per weight at g = 128).
 //
-// Work unit = 16 consecutive weight rows of one matrix over its whole K. Each CTA
-// owns a contiguous range of units, balanced by their number of 128-wide chunks
-// of K (host-computed), so an SM works through one or two matrices at a time and
-// their x stays in L1. Warps take units from the range with a shared-memory
-// counter. A warp streams its units as a flat sequence of chunks: the codes of a
-// chunk (16 rows x 32 bytes) are one 16-byte cp.async per lane, zero-filled past
-// the matrix, into a per-warp ring of kDepth chunks (~128 KB per SM in flight
-// without holding registers); a per-warp queue hands the units claimed by the
-// prefetch cursor to the consuming cursor.
+// Work unit = a block of 256 consecutive weight rows of one matrix over its
+// whole K. Per CTA (one per SM) a producer warp claims units one at a time from
+// a per-launch global counter, in order, with the matrices of the batch sorted
+// by decreasing K (the last units claimed are the shortest; SMs do not all
+// receive HBM data at the same rate, so static shares leave SMs idle). It
+// streams each unit as segments of 256 rows x 512 k: the 32 KB of codes are one
+// 2-D TMA load of 128-byte rows with the 128-byte swizzle (which halves the
+// consumers' bank conflicts; rows past n and columns past k read as zero;
+// narrower rows cost the TMA unit as much per row and halved the stream rate),
+// and the scales of the segment's groups a second 2-D TMA load of a box of 256
+// rows x max(4, 512/g)
+// groups that contains them (re-read from L2 by the segments sharing it; when the
+// scale rows are not a multiple of 16 bytes the producer's 32 lanes copy them
+// with 4-byte cp.async instead), both completing on the segment's "full"
+// mbarrier. TMA keeps a ring of stages
+// segments (~100 KB per SM) in flight without holding registers or load-unit
+// slots — per-lane cp.async streaming tops out near half of HBM bandwidth here.
 //
-// Per chunk a warp runs eight mma.sync.m16n8k16 (bf16 in, fp32 accumulate) with
-// the expanded weights as the 16 x 16 A operand and up to 8 tokens as the n8 B
-// operand (two B tiles for 9..16 tokens), in two independent accumulator chains.
-// The reduction index of the MMA is permuted identically on both operands so that
-// lane (g, t) (g = lane / 4, t = lane % 4) consumes exactly code words 2t, 2t+1 of
-// the chunk for rows g and g + 8 — reduction offsets 32t .. 32t + 31 — and the
-// contiguous 64 bytes x[token g][32t .. 32t + 31]: MMA kb takes offsets
-// 32t + 4kb + {0,1} for fragment slots (2t, 2t+1) and 32t + 4kb + {2,3} for slots
-// (2t+8, 2t+9).
+// Consumer warps own 32 rows of the block (two m16 row tiles that share every
+// activation fragment) over the whole K, so their accumulators persist across the
+// unit's segments; up to 8 tokens two warps share each 32-row slice (each takes
+// half of every segment's chunks, four consumer warps per scheduler) and add
+// their partial sums once per unit through shared memory.
+// Per 128-wide chunk of a segment (four per segment) a warp runs eight
+// mma.sync.m16n8k16 (bf16 in, fp32 accumulate) per row tile with the expanded
+// weights as the 16 x 16 A operand and up to 8 tokens as the n8 B operand (two B
+// tiles for 9..16 tokens). The reduction index of the MMA is permuted identically on both
+// operands so that lane (g, t) (g = lane / 4, t = lane % 4) consumes exactly code
+// words 2t, 2t+1 of the chunk for rows g and g + 8 and the contiguous 64 bytes
+// x[token g][32t .. 32t + 31]: MMA kb takes offsets 32t + 4kb + {0,1} for
+// fragment slots (2t, 2t+1) and 32t + 4kb + {2,3} for slots (2t+8, 2t+9). Tokens
+// past m read token m - 1: their output columns are never stored, and MMA
+// columns do not mix.
 //
 // Expansion: pair j of a code word -> bf16x2 (2c, 2c) by ((w << (14 - 2j)) &
-// 0xC000C000) (layout of include/tq.h). For g >= 128 a chunk lies in one group and
-// the partial sums of a group are scaled by s/2 in fp32 (exact scale); for g <= 64
-// the groups of a chunk meet inside one MMA, so the expansion multiplies by
-// bf16(s)/2 as the prefill kernels do.
+// 0xC000C000) (layout of include/tq.h). For g >= 128 a chunk lies in one group:
+// each group's products are accumulated from zero and folded into the output
+// with the exact fp32 factor s/2. For g <= 64 the groups of a chunk meet inside
+// one MMA, so the expansion multiplies by bf16(s)/2 as the prefill kernels do.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <algorithm>
+#include <atomic>
+
 #include "kernels.cuh"
+#include "ptx.cuh"
 
 namespace tq {
 namespace {
 
-constexpr int kWarps = 16;
-constexpr int kThreads = kWarps * 32;
-constexpr int kDepth = 16;                 // chunks in flight per warp
-constexpr int kChunkBytes = 16 * 32;       // 16 rows x 8 code words
-constexpr int kQueue = kDepth + 1;         // units claimed ahead of the consumer
-constexpr int kSmemBytes = kWarps * kDepth * kChunkBytes;
+constexpr int kRows = kDecodeRows;               // rows per unit (16 per consumer warp)
+constexpr int kTiles = 2;                          // m16 row tiles per consumer warp
+constexpr int kRowWarps = kRows / (16 * kTiles);   // warps covering the unit's rows
+// Up to 8 tokens two warps share each 32-row slice, one per half of every
+// segment's chunks (four consumer warps per scheduler); 9..16 tokens need the
+// registers of one warp per slice.
+template <bool kTwoTiles>
+struct DecodeCfg {
+  static constexpr int kSplit = kTwoTiles ? 1 : 2;
+  static constexpr int kConsumers = kRowWarps * kSplit;
+  static constexpr int kThreads = (kConsumers + 1) * 32;  // + one producer warp
+};
+constexpr int kRedBytes = 2 * kRowWarps * 32 * kTiles * 4 * 4;  // partial sums, two units
+constexpr int kSegK = kDecodeSegK;               // k per segment (one TMA box of 32 words)
+constexpr int kChunks = kSegK / 128;             // 128-wide chunks per segment
+constexpr int kCodeBytes = kRows * kSegK / 4;    // 32 KB
+constexpr int kXRowBytes = kSegK * 2;            // one token's bf16 slice of the segment
+constexpr int kMaxStages = 8;
+constexpr int kHeadBytes = 1024;                 // barriers and segment descriptors
+constexpr int kSmemLimit = 227 * 1024;
+// Slot layout (sizes set per launch from the batch's group sizes and m):
+// [codes 32 KB][scales: 256 rows x (box or segment) groups][x: m tokens x kSegK]
+
+static_assert(kRowWarps == 8, "two m16 row tiles per row warp");
+static_assert(kCodeBytes == 32 * 1024, "codes box");
+
+// Segment descriptor written by the producer next to the slot's barriers; it
+// carries what the consumers need of the matrix, so they never index the
+// parameter table.
+struct SegInfo {
+  int32_t mat;    // matrix of the batch; -1: end of the stream
+  int32_t row0;   // first row of the unit
+  int32_t seg;    // segment index along k
+  int32_t last;   // last segment of the unit
+  int32_t k;      // reduction length
+  int32_t n;      // rows of the matrix
+  int32_t log2g;
+  int32_t mode;   // scale fetch mode | y_bf16 << 8
+  void* y;        // output [m][n]
+  int64_t pad;
+};
+static_assert(sizeof(SegInfo) == 48, "segment descriptor");
 
 __device__ __forceinline__ uint32_t bmul2(uint32_t a, uint32_t b) {
   uint32_t d;
@@ -74,20 +128,33 @@ __device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// 16-byte global -> shared copy; bytes beyond src_bytes (0 or 16) are zero-filled.
+// The same with a zero accumulator input (the first product of a group).
+__device__ __forceinline__ void mma16816_zc(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                            uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+      "{%4, %5, %6, %7}, {%8, %9}, {%10, %10, %10, %10};"
+      : "=f"(c[0]), "=f"(c[1]), "=f"(c[2]), "=f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(0.0f));
+}
+
+// 16-byte global -> shared copy (L2 only); zero-filled when src_bytes is 0.
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
                "r"(src_bytes)
                : "memory");
 }
 
-__device__ __forceinline__ void cp_async_commit() {
-  asm volatile("cp.async.commit_group;" ::: "memory");
+// 4-byte global -> shared copy; zero-filled when src_bytes is 0.
+__device__ __forceinline__ void cp_async4(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(src_bytes)
+               : "memory");
 }
 
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+// Arrive on `bar` once every cp.async this thread issued so far has landed; the
+// arrival counts toward the barrier's expected count.
+__device__ __forceinline__ void cp_async_arrive(uint32_t bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
 }
 
 __device__ __forceinline__ uint32_t half_scale_bf16x2(float s) {
@@ -106,259 +173,491 @@ __device__ __forceinline__ int find_mat(const DecodeBatch& b, int u) {
   return lo;
 }
 
+// Unit scheduler of one launch: {next unit, CTAs done}. Zero at the start of a
+// launch; the last CTA to finish claiming puts both back to zero. Launches take
+// the slots in turn, so up to kSchedSlots launches may be in flight at once.
+constexpr int kSchedSlots = 256;
+__device__ uint32_t g_dsched[kSchedSlots][2];
+
 template <bool kTwoTiles>
-__global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_constant__ DecodeBatch b) {
+__global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
+    decode_kernel(const __grid_constant__ DecodeBatch b, uint32_t* sched) {
+  constexpr int kConsumers = DecodeCfg<kTwoTiles>::kConsumers;
+  constexpr int kSplit = DecodeCfg<kTwoTiles>::kSplit;
   extern __shared__ uint8_t smem_raw[];
-  __shared__ int next_unit;
-  __shared__ int queue[kWarps][kQueue];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) &
-                                             ~static_cast<uintptr_t>(127));
+  uint8_t* head = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const int ub_bytes = b.ubuf_bytes;       // one unit-scale buffer (0: none in this launch)
+  float* red = reinterpret_cast<float*>(head + kHeadBytes);  // [2][kRowWarps][32][8]
+  uint8_t* ubuf = head + kHeadBytes + kRedBytes;             // two unit-scale buffers
+  uint8_t* smem = ubuf + 2 * ub_bytes;     // the ring
+  const int stages = b.stages;
+  const int slot_bytes = b.slot_bytes;
+  const int scale_bytes = b.scale_bytes;
+  const uint32_t ring = smem_u32(smem);
+  const uint32_t bars = smem_u32(head);
+  auto full_bar = [&](int s) { return bars + 8 * s; };
+  auto empty_bar = [&](int s) { return bars + 8 * (kMaxStages + s); };
+  auto sfull_bar = [&](int i) { return bars + 8 * (2 * kMaxStages + i); };
+  auto sempty_bar = [&](int i) { return bars + 8 * (2 * kMaxStages + 2 + i); };
+  // partial-sum hand-off between the two warps of a row slice, per buffer
+  auto rfull_bar = [&](int w, int p) { return bars + 160 + 8 * (2 * w + p); };
+  auto rempty_bar = [&](int w, int p) { return bars + 288 + 8 * (2 * w + p); };
+  SegInfo* info = reinterpret_cast<SegInfo*>(head + 512);  // kMaxStages x 48 bytes
+  int* status = b.status;
+
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int g = lane >> 2, t = lane & 3;
   const int m = b.m;
-  const int uend = b.cta_unit[blockIdx.x + 1];
-  if (threadIdx.x == 0) next_unit = b.cta_unit[blockIdx.x];
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < stages; ++s) {
+      mbar_init(full_bar(s), 1 + 32);  // TMA expect_tx + an arrival per producer lane
+      mbar_init(empty_bar(s), kConsumers);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(sfull_bar(i), 1);
+      mbar_init(sempty_bar(i), kConsumers);
+    }
+    for (int w = 0; w < kRowWarps; ++w)
+      for (int p = 0; p < 2; ++p) {
+        mbar_init(rfull_bar(w, p), 1);
+        mbar_init(rempty_bar(w, p), 1);
+      }
+    fence_mbar_init();
+  }
   __syncthreads();
-  uint8_t* ring = smem + warp * kDepth * kChunkBytes;
-  const uint32_t ring_u32 = static_cast<uint32_t>(__cvta_generic_to_shared(ring));
-  int* q = queue[warp];
+
+  if (warp == kConsumers) {
+    // ------------------------------------------------------------ producer
+    const uint64_t stream_policy = policy_evict_first();  // codes and scales: read once
+    const uint64_t keep_policy = policy_evict_last();     // x: read by every unit
+    int slot = 0;
+    uint32_t parity = 0;
+    int64_t issued = 0;
+    int units_u = 0;  // units whose scales went through the unit buffers
+    bool ok = true;
+    for (;;) {
+      int u = 0;
+      if (lane == 0) u = static_cast<int>(atomicAdd(&sched[0], 1u));
+      u = __shfl_sync(0xffffffffu, u, 0);
+      if (u >= b.total_units) break;
+      const int d = find_mat(b, u);
+      const DecodeMat& mt = b.mats[d];
+      const int64_t row0 = static_cast<int64_t>(u - mt.unit0) * kRows;
+      const int nseg = static_cast<int>((mt.k + kSegK - 1) / kSegK);
+      const int log2g = mt.log2g;
+      const int64_t gpr = mt.k >> log2g;               // groups per row
+      const int ng = log2g >= 9 ? 1 : kSegK >> log2g;  // scales per row per segment
+      if (mt.scale_mode == kDecodeScaleUnit) {
+        // all the unit's scales in one bulk copy (rows past n are not copied;
+        // their outputs are never stored)
+        const int ub = units_u & 1;
+        if (units_u >= 2 && !warp_wait(sempty_bar(ub), ((units_u >> 1) + 1) & 1, status)) {
+          ok = false;
+          break;
+        }
+        if (lane == 0) {
+          const int64_t rows = mt.n - row0 < kRows ? mt.n - row0 : kRows;
+          const uint32_t bytes = static_cast<uint32_t>(rows * gpr * 4);
+          mbar_arrive_expect_tx(sfull_bar(ub), bytes);
+          bulk_load(smem_u32(ubuf + ub * ub_bytes), mt.scales + row0 * gpr, bytes, sfull_bar(ub),
+                    stream_policy);
+        }
+        ++units_u;
+      }
+      for (int s = 0; s < nseg; ++s) {
+        if (issued >= stages && !warp_wait(empty_bar(slot), parity ^ 1u, status)) {
+          ok = false;
+          break;
+        }
+        const int64_t g0 = (static_cast<int64_t>(s) * kSegK) >> log2g;  // first group
+        const uint32_t cdst = ring + slot * slot_bytes;
+        const uint32_t sdst = cdst + kCodeBytes;
+        const uint32_t xdst = sdst + scale_bytes;
+        // the tokens' x over the segment's k (a multiple of 64, so of 128 bytes)
+        const int64_t kx = mt.k - static_cast<int64_t>(s) * kSegK < kSegK
+                               ? mt.k - static_cast<int64_t>(s) * kSegK : kSegK;
+        const uint32_t xbytes = static_cast<uint32_t>(kx) * 2u;
+        if (lane == 0) {
+          info[slot] = SegInfo{d, static_cast<int32_t>(row0), s, s + 1 == nseg ? 1 : 0,
+                               static_cast<int32_t>(mt.k), static_cast<int32_t>(mt.n),
+                               log2g, mt.scale_mode | (mt.y_bf16 << 8), mt.y, 0};
+          mbar_arrive_expect_tx(full_bar(slot), kCodeBytes + static_cast<uint32_t>(m) * xbytes);
+          tma_load_2d_hint(cdst, &b.maps[d], full_bar(slot), s * (kSegK / 16),
+                           static_cast<int32_t>(row0), stream_policy);
+        }
+        __syncwarp();
+        if (lane < m)
+          bulk_load(xdst + lane * kXRowBytes,
+                    static_cast<const __nv_bfloat16*>(mt.x) + lane * mt.k +
+                        static_cast<int64_t>(s) * kSegK,
+                    xbytes, full_bar(slot), keep_policy);
+        if (mt.scale_mode == kDecodeScaleUnit) {
+          mbar_arrive(full_bar(slot));
+        } else {
+          if (mt.scale_mode == kDecodeScale16) {
+            // per row a box of sb groups from a multiple of sb, as 16-byte copies
+            // (k/g % 4 == 0 keeps them aligned), zero past n and past k
+            const int sb = decode_scale_box(log2g);
+            const int64_t gb = g0 - g0 % sb;
+            for (int i = 0; i < kRows / 32; ++i) {
+              const int r = lane + 32 * i;
+              const int64_t row = row0 + r;
+              for (int q = 0; q < sb / 4; ++q) {
+                const bool in = row < mt.n && gb + 4 * q < gpr;
+                const float* src = mt.scales + (in ? row * gpr + gb + 4 * q : 0);
+                cp_async16(sdst + (r * sb + 4 * q) * 4, src, in ? 16u : 0u);
+              }
+            }
+          } else {
+            // [256 rows][ng] from group g0, zero past n and past k
+            for (int i = 0; i < kRows / 32; ++i) {
+              const int r = lane + 32 * i;
+              const int64_t row = row0 + r;
+              for (int q = 0; q < ng; ++q) {
+                const bool in = row < mt.n && g0 + q < gpr;
+                const float* src = mt.scales + (in ? row * gpr + g0 + q : 0);
+                cp_async4(sdst + (r * ng + q) * 4, src, in ? 4u : 0u);
+              }
+            }
+          }
+          cp_async_arrive(full_bar(slot));
+        }
+        ++issued;
+        if (++slot == stages) {
+          slot = 0;
+          parity ^= 1u;
+        }
+      }
+      if (!ok) break;
+    }
+    if (ok) {
+      // end of the stream: a stage with no data tells the consumers
+      if (issued >= stages && !warp_wait(empty_bar(slot), parity ^ 1u, status)) ok = false;
+      if (ok) {
+        if (lane == 0) info[slot].mat = -1;
+        __syncwarp();
+        mbar_arrive(full_bar(slot));  // 32 lanes
+        if (lane == 0) mbar_arrive(full_bar(slot));
+      }
+    }
+    // this CTA claims no more: the last CTA to get here resets the scheduler
+    if (lane == 0) {
+      __threadfence();
+      if (atomicAdd(&sched[1], 1u) == gridDim.x - 1) {
+        atomicExch(&sched[0], 0u);
+        atomicExch(&sched[1], 0u);
+      }
+    }
+    // Nothing may still write this CTA's shared memory when it exits: normally
+    // the consumers waited for every copy; if a wait gave up, wait here for the
+    // segments issued last (no end marker was written on this path) and for the
+    // unit-scale copies.
+    if (!ok && lane == 0) {
+      for (int64_t j = issued > stages ? issued - stages : 0; j < issued; ++j)
+        if (!mbar_wait(full_bar(static_cast<int>(j % stages)),
+                       static_cast<uint32_t>((j / stages) & 1), status))
+          break;
+      for (int j = units_u > 2 ? units_u - 2 : 0; j < units_u; ++j)
+        if (!mbar_wait(sfull_bar(j & 1), (j >> 1) & 1, status)) break;
+    }
+    if (!ok) asm volatile("cp.async.wait_all;" ::: "memory");
+    return;
+  }
+
+  // -------------------------------------------------------------- consumers
+  // Warp w owns rows 32wr .. 32wr + 31 of the unit (wr = w % 8) as two m16 tiles
+  // that share every activation fragment, over the chunks c of each segment with
+  // c / (4 / kSplit) == w / 8; lane (g, t) holds rows 32wr + 16r + g (+8) of tile r.
+  const int wr = warp % kRowWarps;
+  const int kh = warp / kRowWarps;  // which part of every segment's chunks
+  const int g = lane >> 2, t = lane & 3;
   uint32_t mul[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) mul[j] = opaque(1u << (14 - 2 * j));
-
-  // ------------------------------------------------------------ prefetch cursor
-  // Lane l copies 16 bytes per chunk: row l / 2 of the unit, words 4 (l & 1) .. + 3.
-  const int crow = lane >> 1, chalf = lane & 1;
-  int qtail = 0;            // units claimed (queue writes)
-  int pu = -1;              // unit being prefetched (-1: stream exhausted)
-  int pc = 0, pnc = 0;      // its next chunk / chunk count
-  const uint32_t* psrc = nullptr;
-  bool prow = false;        // this lane's row exists
-  bool phalf = false;       // this lane's half of the last chunk lies past k
-  auto claim = [&]() {
-    int u = 0;
-    if (lane == 0) u = atomicAdd(&next_unit, 1);
-    u = __shfl_sync(0xffffffffu, u, 0);
-    if (u >= uend) {
-      pu = -1;
-      return;
-    }
-    const int d = find_mat(b, u);
-    const DecodeMat& mat = b.mats[d];
-    const int64_t row = static_cast<int64_t>(u - mat.unit0) * 16 + crow;
-    pu = u;
-    pc = 0;
-    pnc = static_cast<int>((mat.k + 127) >> 7);
-    prow = row < mat.n;
-    phalf = chalf && (mat.k & 127);
-    psrc = mat.codes + (prow ? row : 0) * (mat.k >> 4) + chalf * 4;
-    if (lane == 0) q[qtail % kQueue] = u;
-    ++qtail;
-  };
-  auto issue = [&](int slot) {
-    if (pu >= 0) {
-      const bool in = prow && !(phalf && pc + 1 == pnc);
-      cp_async16(ring_u32 + slot * kChunkBytes + crow * 32 + chalf * 16, psrc + 8 * pc,
-                 in ? 16u : 0u);
-      if (++pc == pnc) claim();
-    }
-    cp_async_commit();  // one group per slot, empty past the end of the stream
-  };
-
-  claim();
-  for (int s = 0; s < kDepth - 1; ++s) issue(s);
-
-  // ------------------------------------------------------------ consumer
-  int qhead = 0;
-  int slot = 0;
-  while (qhead < qtail) {
-    __syncwarp();
-    const int u = q[qhead % kQueue];
-    ++qhead;
-    const int d = find_mat(b, u);
-    const DecodeMat& mat = b.mats[d];
-    const int64_t n = mat.n, k = mat.k;
-    const int64_t r0 = static_cast<int64_t>(u - mat.unit0) * 16;
-    const int64_t ra = r0 + g, rb = r0 + g + 8;
-    const bool va = ra < n, vb = rb < n;
-    const int log2g = mat.log2g;
-    const int64_t gpr = k >> log2g;
-    const float* sa = mat.scales + (va ? ra : 0) * gpr;
-    const float* sb = mat.scales + (vb ? rb : 0) * gpr;
-    const bool ta = g < m, tb = kTwoTiles && (g + 8 < m);
-    const uint4* xa = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(mat.x) +
-                                                     static_cast<int64_t>(ta ? g : 0) * k + 32 * t);
-    const uint4* xb = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(mat.x) +
-                                                     static_cast<int64_t>(tb ? g + 8 : 0) * k + 32 * t);
-    const int nc = static_cast<int>((k + 127) >> 7);
-    // a lane's 32 offsets of the last chunk lie past k when k % 128 == 64 and t >= 2
-    const bool tail_lane = (k & 127) && t >= 2;
-    float acc0[4] = {0.f, 0.f, 0.f, 0.f}, acc1[4] = {0.f, 0.f, 0.f, 0.f};
-    float p0[4] = {0.f, 0.f, 0.f, 0.f}, p1[4] = {0.f, 0.f, 0.f, 0.f};
-    float q0[4] = {0.f, 0.f, 0.f, 0.f}, q1[4] = {0.f, 0.f, 0.f, 0.f};
-
-    if (log2g >= 7) {
-      // exact path: one scale per row per group of (g / 128) chunks
-      const int cpg = 1 << (log2g - 7);
-      int left = cpg;
-      int gi = 0;
-      for (int c = 0; c < nc; ++c) {
-        issue((slot + kDepth - 1) % kDepth);
-        cp_async_wait<kDepth - 1>();
-        __syncwarp();
-        const uint8_t* st = ring + slot * kChunkBytes;
-        const uint2 wa = *reinterpret_cast<const uint2*>(st + g * 32 + 8 * t);
-        const uint2 wb = *reinterpret_cast<const uint2*>(st + (g + 8) * 32 + 8 * t);
-        uint4 xv[4], yv[4];
+  float acc[kTiles][4], acc1[kTiles][4];  // tokens 0..7 and 8..15
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          xv[i] = ta ? __ldg(xa + 16 * c + i) : make_uint4(0, 0, 0, 0);
-          if (kTwoTiles) yv[i] = tb ? __ldg(xb + 16 * c + i) : make_uint4(0, 0, 0, 0);
-        }
-        const uint32_t* xr = reinterpret_cast<const uint32_t*>(xv);
-        const uint32_t* yr = reinterpret_cast<const uint32_t*>(yv);
+  for (int r = 0; r < kTiles; ++r)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) acc[r][i] = acc1[r][i] = 0.f;
+  const int tok0 = g < m ? g : m - 1;  // tokens past m read token m - 1
+  const int tok1 = g + 8 < m ? g + 8 : m - 1;
+  const int rl = 32 * wr + g;          // row of tile 0 for C slots 0, 1 (+8: slots 2, 3)
+  int units_r = 0;                     // units whose partial sums were handed over
+
+  int slot = 0;
+  uint32_t parity = 0;
+  int units_u = 0;
+  for (;;) {
+    if (!warp_wait(full_bar(slot), parity, status)) return;
+    const SegInfo si = info[slot];
+    if (si.mat < 0) break;
+    const int64_t k = si.k;
+    const int log2g = si.log2g;
+    const int mode = si.mode & 0xff;
+    const int g0 = (si.seg * kSegK) >> log2g;  // first group of the segment
+    const uint8_t* cbase = smem + slot * slot_bytes;
+    // scale of unit row r and group q: sp[r * sstride + q - sq0]
+    const float* sp;
+    int sstride, sq0;
+    const bool unit_scales = mode == kDecodeScaleUnit;
+    if (unit_scales) {
+      const int ub = units_u & 1;
+      if (si.seg == 0 && !warp_wait(sfull_bar(ub), (units_u >> 1) & 1, status)) return;
+      sp = reinterpret_cast<const float*>(ubuf + ub * ub_bytes);
+      sstride = static_cast<int>(k >> log2g);
+      sq0 = 0;
+    } else {
+      sp = reinterpret_cast<const float*>(cbase + kCodeBytes);
+      if (mode == kDecodeScale16) {
+        sstride = decode_scale_box(log2g);
+        sq0 = g0 - g0 % sstride;
+      } else {
+        sstride = log2g >= 9 ? 1 : kSegK >> log2g;
+        sq0 = g0;
+      }
+    }
+    const uint8_t* xs = cbase + kCodeBytes + scale_bytes;  // x [m tokens][kSegK]
+    if (si.seg == 0) {
+#pragma unroll
+      for (int r = 0; r < kTiles; ++r)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[r][i] = acc1[r][i] = 0.f;
+    }
+#pragma unroll
+    for (int cc = 0; cc < kChunks / kSplit; ++cc) {
+      const int c = kh * (kChunks / kSplit) + cc;
+      const int64_t kc = static_cast<int64_t>(si.seg) * kSegK + 128 * c;  // chunk start
+      if (kc >= k) break;
+      const bool kin = kc + 32 * t + 32 <= k;  // this lane's 32 offsets lie inside k
+      // The codes box is 128-byte swizzled: 16-byte chunk j of row r sits at chunk
+      // j ^ (r % 8); every row of this lane has r % 8 = g.
+      const int co = (((2 * c + (t >> 1)) ^ g) << 4) + (t & 1) * 8;
+      uint2 w[kTiles][2];
+#pragma unroll
+      for (int r = 0; r < kTiles; ++r) {
+        const uint8_t* cw = cbase + (rl + 16 * r) * (kSegK / 4) + co;
+        w[r][0] = *reinterpret_cast<const uint2*>(cw);
+        w[r][1] = *reinterpret_cast<const uint2*>(cw + 8 * (kSegK / 4));
+      }
+      // past k (a lane of a half chunk) the slot holds no x
+      uint4 xv[4], yv[4];
+      const int xo = (128 * c + 32 * t) * 2;
+      const uint4* xa = reinterpret_cast<const uint4*>(xs + tok0 * kXRowBytes + xo);
+      const uint4* xb = reinterpret_cast<const uint4*>(xs + tok1 * kXRowBytes + xo);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        xv[i] = kin ? xa[i] : make_uint4(0, 0, 0, 0);
+        if (kTwoTiles) yv[i] = kin ? xb[i] : make_uint4(0, 0, 0, 0);
+      }
+      const uint32_t* xr = reinterpret_cast<const uint32_t*>(xv);
+      const uint32_t* yr = reinterpret_cast<const uint32_t*>(yv);
+      if (log2g >= 7) {
+        // exact path: the chunk lies in one group; its products are accumulated
+        // from zero and folded in with the fp32 factor s/2 of that group
+        float p[kTiles][4], p1[kTiles][4];
 #pragma unroll
         for (int kb = 0; kb < 8; ++kb) {
-          const uint32_t ua = kb < 4 ? wa.x : wa.y, ub = kb < 4 ? wb.x : wb.y;
           const int j = 2 * (kb & 3);
-          const uint32_t a0 = pair_bits(ua, j, mul[j]), a1 = pair_bits(ub, j, mul[j]);
-          const uint32_t a2 = pair_bits(ua, j + 1, mul[j + 1]), a3 = pair_bits(ub, j + 1, mul[j + 1]);
-          if (kb & 1) {
-            mma16816(q0, a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
-            if (kTwoTiles) mma16816(q1, a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
-          } else {
-            mma16816(p0, a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
-            if (kTwoTiles) mma16816(p1, a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
-          }
-        }
-        __syncwarp();
-        slot = slot + 1 == kDepth ? 0 : slot + 1;
-        if (--left == 0) {
-          // group closed: acc += (s / 2) * partial; rows g (slots 0, 1), g + 8 (2, 3)
-          left = cpg;
-          const float ha = va ? 0.5f * __ldg(sa + gi) : 0.f;
-          const float hb = vb ? 0.5f * __ldg(sb + gi) : 0.f;
-          ++gi;
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const float h = i < 2 ? ha : hb;
-            acc0[i] = fmaf(h, p0[i] + q0[i], acc0[i]);
-            p0[i] = q0[i] = 0.f;
-            if (kTwoTiles) {
-              acc1[i] = fmaf(h, p1[i] + q1[i], acc1[i]);
-              p1[i] = q1[i] = 0.f;
+          for (int r = 0; r < kTiles; ++r) {
+            const uint32_t u0 = kb < 4 ? w[r][0].x : w[r][0].y;
+            const uint32_t u1 = kb < 4 ? w[r][1].x : w[r][1].y;
+            const uint32_t a0 = pair_bits(u0, j, mul[j]), a1 = pair_bits(u1, j, mul[j]);
+            const uint32_t a2 = pair_bits(u0, j + 1, mul[j + 1]);
+            const uint32_t a3 = pair_bits(u1, j + 1, mul[j + 1]);
+            if (kb == 0) {
+              mma16816_zc(p[r], a0, a1, a2, a3, xr[0], xr[1]);
+              if (kTwoTiles) mma16816_zc(p1[r], a0, a1, a2, a3, yr[0], yr[1]);
+            } else {
+              mma16816(p[r], a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
+              if (kTwoTiles) mma16816(p1[r], a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
             }
           }
         }
-      }
-    } else {
-      // g = 32 or 64: lane t's offsets 32t .. 32t + 31 of a chunk lie in one group
-      const int gshift = 7 - log2g;  // groups per chunk = 1 << gshift
-      for (int c = 0; c < nc; ++c) {
-        issue((slot + kDepth - 1) % kDepth);
-        cp_async_wait<kDepth - 1>();
-        __syncwarp();
-        const bool kin = !(tail_lane && c + 1 == nc);
-        const uint8_t* st = ring + slot * kChunkBytes;
-        const uint2 wa = *reinterpret_cast<const uint2*>(st + g * 32 + 8 * t);
-        const uint2 wb = *reinterpret_cast<const uint2*>(st + (g + 8) * 32 + 8 * t);
-        const int64_t gi = (static_cast<int64_t>(c) << gshift) + (t >> (log2g - 5));
-        const uint32_t ha = (va && kin) ? half_scale_bf16x2(__ldg(sa + gi)) : 0u;
-        const uint32_t hb = (vb && kin) ? half_scale_bf16x2(__ldg(sb + gi)) : 0u;
-        uint4 xv[4], yv[4];
+        // C slots 0, 1: row rl + 16r, slots 2, 3: row rl + 16r + 8
+        const int q = static_cast<int>(kc >> log2g) - sq0;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          xv[i] = (ta && kin) ? __ldg(xa + 16 * c + i) : make_uint4(0, 0, 0, 0);
-          if (kTwoTiles) yv[i] = (tb && kin) ? __ldg(xb + 16 * c + i) : make_uint4(0, 0, 0, 0);
-        }
-        const uint32_t* xr = reinterpret_cast<const uint32_t*>(xv);
-        const uint32_t* yr = reinterpret_cast<const uint32_t*>(yv);
+        for (int r = 0; r < kTiles; ++r) {
+          const float h0 = 0.5f * sp[(rl + 16 * r) * sstride + q];
+          const float h1 = 0.5f * sp[(rl + 16 * r + 8) * sstride + q];
 #pragma unroll
-        for (int kb = 0; kb < 8; ++kb) {
-          const uint32_t ua = kb < 4 ? wa.x : wa.y, ub = kb < 4 ? wb.x : wb.y;
-          const int j = 2 * (kb & 3);
-          const uint32_t a0 = bmul2(pair_bits(ua, j, mul[j]), ha), a1 = bmul2(pair_bits(ub, j, mul[j]), hb);
-          const uint32_t a2 = bmul2(pair_bits(ua, j + 1, mul[j + 1]), ha), a3 = bmul2(pair_bits(ub, j + 1, mul[j + 1]), hb);
-          if (kb & 1) {
-            mma16816(q0, a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
-            if (kTwoTiles) mma16816(q1, a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
-          } else {
-            mma16816(acc0, a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
-            if (kTwoTiles) mma16816(acc1, a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
+          for (int i = 0; i < 4; ++i) {
+            acc[r][i] = fmaf(i < 2 ? h0 : h1, p[r][i], acc[r][i]);
+            if (kTwoTiles) acc1[r][i] = fmaf(i < 2 ? h0 : h1, p1[r][i], acc1[r][i]);
           }
         }
-        __syncwarp();
-        slot = slot + 1 == kDepth ? 0 : slot + 1;
-      }
+      } else {
+        // g = 32 or 64: lane t's offsets 32t .. 32t + 31 of a chunk lie in one
+        // group, whose bf16(s)/2 multiplies the expanded pairs
+        const int q = static_cast<int>((kc + 32 * t) >> log2g) - sq0;
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        acc0[i] += q0[i];
-        if (kTwoTiles) acc1[i] += q1[i];
+        for (int r = 0; r < kTiles; ++r) {
+          const uint32_t hs0 = kin ? half_scale_bf16x2(sp[(rl + 16 * r) * sstride + q]) : 0u;
+          const uint32_t hs1 = kin ? half_scale_bf16x2(sp[(rl + 16 * r + 8) * sstride + q]) : 0u;
+#pragma unroll
+          for (int kb = 0; kb < 8; ++kb) {
+            const int j = 2 * (kb & 3);
+            const uint32_t u0 = kb < 4 ? w[r][0].x : w[r][0].y;
+            const uint32_t u1 = kb < 4 ? w[r][1].x : w[r][1].y;
+            const uint32_t a0 = bmul2(pair_bits(u0, j, mul[j]), hs0);
+            const uint32_t a1 = bmul2(pair_bits(u1, j, mul[j]), hs1);
+            const uint32_t a2 = bmul2(pair_bits(u0, j + 1, mul[j + 1]), hs0);
+            const uint32_t a3 = bmul2(pair_bits(u1, j + 1, mul[j + 1]), hs1);
+            mma16816(acc[r], a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
+            if (kTwoTiles) mma16816(acc1[r], a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
+          }
+        }
       }
     }
-
-    // C fragment: rows g (slots 0, 1) and g + 8 (slots 2, 3), tokens 2t and 2t + 1
-    auto store = [&](int token, int64_t row, float v) {
-      if (token < m && row < n) {
-        if (mat.y_bf16)
-          static_cast<__nv_bfloat16*>(mat.y)[token * n + row] = __float2bfloat16_rn(v);
-        else
-          static_cast<float*>(mat.y)[token * n + row] = v;
+    __syncwarp();
+    if (lane == 0) {
+      mbar_arrive(empty_bar(slot));
+      if (unit_scales && si.last) mbar_arrive(sempty_bar(units_u & 1));
+    }
+    if (unit_scales && si.last) ++units_u;
+    if (si.last && kSplit == 2) {
+      // the second warp of the slice hands its partial sums to the first through
+      // buffer units_r % 2 (bounded waits both ways: "written" and "read")
+      const int pb = units_r & 1;
+      const uint32_t ph = (units_r >> 1) & 1;
+      float* rb = red + ((pb * kRowWarps + wr) * 32 + lane) * (kTiles * 4);
+      if (kh == 1) {
+        if (units_r >= 2 && !warp_wait(rempty_bar(wr, pb), ph ^ 1u, status)) return;
+#pragma unroll
+        for (int r = 0; r < kTiles; ++r)
+#pragma unroll
+          for (int i = 0; i < 4; ++i) rb[r * 4 + i] = acc[r][i];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(rfull_bar(wr, pb));
+      } else {
+        if (!warp_wait(rfull_bar(wr, pb), ph, status)) return;
+#pragma unroll
+        for (int r = 0; r < kTiles; ++r)
+#pragma unroll
+          for (int i = 0; i < 4; ++i) acc[r][i] += rb[r * 4 + i];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(rempty_bar(wr, pb));
       }
-    };
-    store(2 * t, ra, acc0[0]);
-    store(2 * t + 1, ra, acc0[1]);
-    store(2 * t, rb, acc0[2]);
-    store(2 * t + 1, rb, acc0[3]);
-    if (kTwoTiles) {
-      store(8 + 2 * t, ra, acc1[0]);
-      store(8 + 2 * t + 1, ra, acc1[1]);
-      store(8 + 2 * t, rb, acc1[2]);
-      store(8 + 2 * t + 1, rb, acc1[3]);
+      ++units_r;
+    }
+    if (si.last && kh == 0) {
+      // C fragment of tile r: rows rl + 16r (slots 0, 1) and + 8 (2, 3), tokens 2t, 2t + 1
+      const int64_t n = si.n;
+      const bool ybf16 = (si.mode >> 8) != 0;
+      auto store = [&](int token, int64_t row, float v) {
+        if (token < m && row < n) {
+          if (ybf16)
+            static_cast<__nv_bfloat16*>(si.y)[token * n + row] = __float2bfloat16_rn(v);
+          else
+            static_cast<float*>(si.y)[token * n + row] = v;
+        }
+      };
+#pragma unroll
+      for (int r = 0; r < kTiles; ++r) {
+        const int64_t ra = si.row0 + rl + 16 * r, rb = ra + 8;
+        store(2 * t, ra, acc[r][0]);
+        store(2 * t + 1, ra, acc[r][1]);
+        store(2 * t, rb, acc[r][2]);
+        store(2 * t + 1, rb, acc[r][3]);
+        if (kTwoTiles) {
+          store(8 + 2 * t, ra, acc1[r][0]);
+          store(8 + 2 * t + 1, ra, acc1[r][1]);
+          store(8 + 2 * t, rb, acc1[r][2]);
+          store(8 + 2 * t + 1, rb, acc1[r][3]);
+        }
+      }
+    }
+    if (++slot == stages) {
+      slot = 0;
+      parity ^= 1u;
     }
   }
-  cp_async_wait<0>();  // nothing may still write this warp's ring when it exits
+}
+
+// Device address of g_dsched, looked up once per device.
+uint32_t* dsched_base() {
+  static std::atomic<uintptr_t> base[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+  if (dev < 64) {
+    const uintptr_t p = base[dev].load(std::memory_order_acquire);
+    if (p != 0) return reinterpret_cast<uint32_t*>(p);
+  }
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_dsched) != cudaSuccess) return nullptr;
+  if (dev < 64) base[dev].store(reinterpret_cast<uintptr_t>(p), std::memory_order_release);
+  return static_cast<uint32_t*>(p);
 }
 
 }  // namespace
 
 cudaError_t launch_decode(DecodeBatch& b, int num_sms, cudaStream_t stream) {
-  if (b.total_units <= 0) return cudaSuccess;
-  int64_t blocks = (static_cast<int64_t>(b.total_units) + kWarps - 1) / kWarps;
-  if (blocks > num_sms) blocks = num_sms;
-  if (blocks > kDecodeMaxCtas) blocks = kDecodeMaxCtas;
-  // Split the units into `blocks` contiguous ranges of about equal chunk count.
-  int64_t work = 0;
-  for (int d = 0; d < b.count; ++d) {
-    const int64_t units = (b.mats[d].n + 15) / 16;
-    work += units * ((b.mats[d].k + 127) / 128);
-  }
-  int c = 0;
-  int64_t acc = 0;
-  b.cta_unit[0] = 0;
-  for (int d = 0; d < b.count && c + 1 < blocks; ++d) {
-    const int64_t units = (b.mats[d].n + 15) / 16;
-    const int64_t per = (b.mats[d].k + 127) / 128;
-    for (int64_t u = 0; u < units && c + 1 < blocks; ++u) {
-      acc += per;
-      // close range c once it holds its share (c + 1) * work / blocks
-      while (c + 1 < blocks && acc * blocks >= (c + 1) * work) {
-        b.cta_unit[++c] = b.mats[d].unit0 + static_cast<int32_t>(u) + 1;
-      }
+  static std::atomic<uint32_t> seq{0};
+  // longest rows first: the units claimed last are the shortest (matrices and
+  // their tensor maps move together)
+  int order[kDecodeMaxMats];
+  for (int d = 0; d < b.count; ++d) order[d] = d;
+  std::stable_sort(order, order + b.count,
+                   [&](int x, int y) { return b.mats[x].k > b.mats[y].k; });
+  bool sorted = true;
+  for (int d = 0; d < b.count; ++d) sorted = sorted && order[d] == d;
+  if (!sorted) {
+    static thread_local DecodeBatch tmp;
+    for (int d = 0; d < b.count; ++d) {
+      tmp.mats[d] = b.mats[order[d]];
+      tmp.maps[d] = b.maps[order[d]];
+    }
+    for (int d = 0; d < b.count; ++d) {
+      b.mats[d] = tmp.mats[d];
+      b.maps[d] = tmp.maps[d];
     }
   }
-  while (c < blocks) b.cta_unit[++c] = b.total_units;
-  const size_t smem = kSmemBytes + 128;
+  int64_t units = 0;
+  for (int d = 0; d < b.count; ++d) {
+    b.mats[d].unit0 = static_cast<int32_t>(units);
+    units += (b.mats[d].n + kRows - 1) / kRows;
+  }
+  if (units >= (int64_t{1} << 31)) return cudaErrorInvalidValue;
+  b.total_units = static_cast<int32_t>(units);
+  if (b.total_units <= 0) return cudaSuccess;
+  const int64_t blocks = units < num_sms ? units : num_sms;
+  // unit-scale buffers: the largest unit of scales among unit-mode matrices;
+  // ring slot: codes + the widest per-segment scale area + x of the m tokens
+  int64_t ugroups = 0;
+  int sgroups = 0;
+  for (int d = 0; d < b.count; ++d) {
+    const int lg = b.mats[d].log2g;
+    const int64_t gpr = b.mats[d].k >> lg;
+    if (b.mats[d].scale_mode == kDecodeScaleUnit) {
+      ugroups = gpr > ugroups ? gpr : ugroups;
+    } else {
+      const int w = b.mats[d].scale_mode == kDecodeScale16 ? decode_scale_box(lg) : (lg >= 9 ? 1 : kSegK >> lg);
+      sgroups = w > sgroups ? w : sgroups;
+    }
+  }
+  b.ubuf_bytes = static_cast<int32_t>(kRows * ugroups * 4);
+  b.scale_bytes = kRows * sgroups * 4;
+  b.slot_bytes = (kCodeBytes + b.scale_bytes + b.m * kXRowBytes + 1023) & ~1023;
+  const int fit = (kSmemLimit - 1024 - kHeadBytes - kRedBytes - 2 * b.ubuf_bytes) / b.slot_bytes;
+  b.stages = fit < kMaxStages ? fit : kMaxStages;
+  if (b.stages < 2) return cudaErrorInvalidValue;
+  const int smem = 1024 + kHeadBytes + kRedBytes + 2 * b.ubuf_bytes + b.stages * b.slot_bytes;
+  uint32_t* sched = dsched_base();
+  if (sched == nullptr) return cudaErrorInvalidSymbol;
+  sched += 2 * (seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
   cudaError_t e;
   if (b.m > 8) {
-    e = ensure_smem_limit<decode_kernel<true>>(static_cast<int>(smem));
+    e = ensure_smem_limit<decode_kernel<true>>(kSmemLimit);
     if (e != cudaSuccess) return e;
-    decode_kernel<true><<<static_cast<unsigned>(blocks), kThreads, smem, stream>>>(b);
+    decode_kernel<true><<<static_cast<unsigned>(blocks), DecodeCfg<true>::kThreads, smem, stream>>>(
+        b, sched);
   } else {
-    e = ensure_smem_limit<decode_kernel<false>>(static_cast<int>(smem));
+    e = ensure_smem_limit<decode_kernel<false>>(kSmemLimit);
     if (e != cudaSuccess) return e;
-    decode_kernel<false><<<static_cast<unsigned>(blocks), kThreads, smem, stream>>>(b);
+    decode_kernel<false><<<static_cast<unsigned>(blocks), DecodeCfg<false>::kThreads, smem,
+                           stream>>>(b, sched);
   }
   return cudaGetLastError();
 }

@@ -87,30 +87,44 @@ cudaError_t launch_ts_gemm(int mode, int bn, const CUtensorMap& tmap_b,
 // decode.cu ------------------------------------------------------------------
 // Forward for m <= 16 tokens over one or many matrices in one launch.
 struct DecodeMat {
-  const uint32_t* codes;  // uint32 [n][k/16]
   const float* scales;    // fp32 [n][k/g]
   const void* x;          // bf16 [m][k]
   void* y;                // [m][n], fp32 or bf16
   int64_t n, k;           // k % 64 == 0
   int32_t log2g;
   int32_t y_bf16;
-  int32_t unit0;          // first 16-row unit of this matrix in the batch
-  int32_t pad;
+  int32_t unit0;          // first unit of this matrix in the batch (set by the launcher)
+  int32_t scale_mode;     // how the kernel fetches scales (host-set, kDecodeScale*)
 };
 
-constexpr int kDecodeMaxMats = 256;
-constexpr int kDecodeMaxCtas = 256;
+// Scale fetch modes: per segment in 4-byte pieces; per segment in 16-byte pieces
+// (k/g % 4 == 0); a whole unit in one bulk copy (k/g % 4 == 0, k/g <= 32).
+constexpr int kDecodeScale4 = 0, kDecodeScale16 = 1, kDecodeScaleUnit = 2;
+constexpr int kDecodeMaxMats = 128;  // per launch (the tensor maps travel as parameters)
+constexpr int kDecodeRows = 256;    // weight rows per work unit
+constexpr int kDecodeSegK = 512;    // k per streamed segment (128-byte code rows)
+
+// Groups per row of a decode scale box: kDecodeSegK / g, at least 4 (16 bytes).
+__host__ __device__ constexpr int decode_scale_box(int log2g) {
+  return (kDecodeSegK >> log2g) > 4 ? (kDecodeSegK >> log2g) : 4;
+}
 
 struct DecodeBatch {
+  // codes of matrix d as uint32 [n][k/16], box {kDecodeSegK / 16 words, kDecodeRows rows},
+  // 128-byte swizzle
+  CUtensorMap maps[kDecodeMaxMats];
   DecodeMat mats[kDecodeMaxMats];
-  int32_t cta_unit[kDecodeMaxCtas + 1];  // CTA c owns units [cta_unit[c], cta_unit[c + 1])
   int* status;            // device status word (timeouts)
   int32_t count;
   int32_t m;              // tokens, 1..16
-  int32_t total_units;    // sum over matrices of ceil(n / 16)
-  int32_t pad;
+  int32_t total_units;    // sum over matrices of ceil(n / kDecodeRows) (set by the launcher)
+  int32_t slot_bytes;     // shared-memory ring slot: codes, scales, x (set by the launcher)
+  int32_t scale_bytes;    // scale area of a slot
+  int32_t stages;         // ring slots
+  int32_t ubuf_bytes;     // one unit-scale buffer (two are kept)
 };
 
+// Reorders b.mats / b.maps (decreasing k) and sets unit0 and total_units.
 cudaError_t launch_decode(DecodeBatch& batch, int num_sms, cudaStream_t stream);
 
 // dw_gemm.cu -----------------------------------------------------------------

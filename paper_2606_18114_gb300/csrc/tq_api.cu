@@ -12,6 +12,7 @@
 #include <string.h>
 
 #include <mutex>
+#include <unordered_map>
 
 #include "kernels.cuh"
 #include "tq.h"
@@ -183,17 +184,76 @@ tq_status fwd_checked(const void* x, int64_t m, int64_t k, const uint32_t* codes
   return e == cudaSuccess ? TQ_OK : cuda_fail(e, "forward launch");
 }
 
-static_assert(tq::kDecodeMaxMats >= TQ_MAX_BATCH, "decode batch table");
 static_assert(tq::kQuantMaxMats >= TQ_MAX_BATCH, "quantize batch table");
 
-// Forward for m <= 16 tokens: the HBM-streaming decode kernel over all matrices.
+// Tensor map of a codes matrix for the decode kernel, cached by (device, codes,
+// n, k): a map encodes only the address, shape and strides, so a cached entry
+// stays right for as long as the same call can be made again.
+struct MapKey {
+  int dev;
+  const void* codes;
+  int64_t n, k;
+  bool operator==(const MapKey& o) const {
+    return dev == o.dev && codes == o.codes && n == o.n && k == o.k;
+  }
+};
+struct MapKeyHash {
+  size_t operator()(const MapKey& x) const {
+    size_t h = std::hash<const void*>()(x.codes);
+    h ^= std::hash<int64_t>()(x.n) + 0x9e3779b97f4a7c15ull + (h << 6) + (h >> 2);
+    h ^= std::hash<int64_t>()(x.k) + 0x9e3779b97f4a7c15ull + (h << 6) + (h >> 2);
+    return h ^ static_cast<size_t>(x.dev);
+  }
+};
+
+// kind 0: codes uint32 [n][k/16]; kind 1: scales fp32 [n][k/g] (k here = k/g) with
+// a box of `box` groups.
+tq_status decode_map(int kind, const void* base, int64_t n, int64_t k, uint32_t box,
+                     CUtensorMap* out) {
+  static std::mutex mu;
+  static std::unordered_map<MapKey, CUtensorMap, MapKeyHash> cache;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  const MapKey key{dev * 2 + kind, base, n, k * 1024 + box};
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    auto it = cache.find(key);
+    if (it != cache.end()) {
+      *out = it->second;
+      return TQ_OK;
+    }
+  }
+  if (kind == 0)
+    TQ_TRY(make_map(out, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, base, k / 16, n,
+                    tq::kDecodeSegK / 16, tq::kDecodeRows, CU_TENSOR_MAP_SWIZZLE_128B));
+  else
+    TQ_TRY(make_map(out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, base, k, n, box, tq::kDecodeRows,
+                    CU_TENSOR_MAP_SWIZZLE_NONE));
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache.size() >= 4096) cache.clear();
+  cache.emplace(key, *out);
+  return TQ_OK;
+}
+
+// Forward for m <= 16 tokens: the HBM-streaming decode kernel over all matrices
+// (launches of up to kDecodeMaxMats matrices each).
 tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
                          cudaStream_t stream) {
   const DeviceInfo* dev = nullptr;
   TQ_TRY(device_info(&dev));
   thread_local tq::DecodeBatch b;
-  int64_t units = 0;
   int used = 0;
+  auto flush = [&]() -> tq_status {
+    if (used == 0) return TQ_OK;
+    b.status = dev->status;
+    b.count = used;
+    b.m = static_cast<int32_t>(m);
+    b.total_units = 0;
+    used = 0;
+    cudaError_t e = tq::launch_decode(b, dev->num_sms, stream);
+    return e == cudaSuccess ? TQ_OK : cuda_fail(e, "decode launch");
+  };
   for (int32_t i = 0; i < count; ++i) {
     const tq_fwd_desc& d = descs[i];
     if (d.n == 0) continue;
@@ -203,26 +263,25 @@ tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
       if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
       continue;
     }
+    if (d.n >= (int64_t(1) << 31)) return fail(TQ_ERR_UNSUPPORTED, "too many decode rows");
+    const int log2g = log2_group(d.g);
+    const int64_t gpr = d.k >> log2g;
+    TQ_TRY(decode_map(0, d.codes, d.n, d.k, 0, &b.maps[used]));
     tq::DecodeMat& dm = b.mats[used++];
-    dm.codes = d.codes;
     dm.scales = d.scales;
     dm.x = d.x;
     dm.y = d.y;
     dm.n = d.n;
     dm.k = d.k;
-    dm.log2g = log2_group(d.g);
+    dm.log2g = log2g;
     dm.y_bf16 = d.y_dtype == TQ_OUT_BF16;
-    dm.unit0 = static_cast<int32_t>(units);
-    units += (d.n + 15) / 16;
-    if (units >= (int64_t(1) << 31)) return fail(TQ_ERR_UNSUPPORTED, "too many decode rows");
+    dm.unit0 = 0;
+    dm.scale_mode = gpr % 4 != 0 ? tq::kDecodeScale4
+                    : gpr <= 32  ? tq::kDecodeScaleUnit
+                                 : tq::kDecodeScale16;
+    if (used == tq::kDecodeMaxMats) TQ_TRY(flush());
   }
-  if (used == 0) return TQ_OK;
-  b.status = dev->status;
-  b.count = used;
-  b.m = static_cast<int32_t>(m);
-  b.total_units = static_cast<int32_t>(units);
-  cudaError_t e = tq::launch_decode(b, dev->num_sms, stream);
-  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "decode launch");
+  return flush();
 }
 
 tq_status check_fwd_args(const void* x, int64_t m, int64_t k, const uint32_t* codes,
