@@ -197,11 +197,11 @@ class Prefill:
 
 
 KERNELS = [  # name, source files, event span
-    ("quantize", ["quantize.cu"], (0, 1)),
-    ("transpose", ["quantize.cu"], (1, 2)),
-    ("fwd", ["ts_gemm.cu", "ptx.cuh"], (2, 3)),
-    ("dx", ["ts_gemm.cu", "ptx.cuh"], (3, 4)),
-    ("dw", ["dw_gemm.cu", "ptx.cuh"], (4, 5)),
+    ("quantize", ["quantize.cu", "ptx.cuh", "kernels.cuh"], (0, 1)),
+    ("transpose", ["quantize.cu", "kernels.cuh"], (1, 2)),
+    ("fwd", ["ts_gemm.cu", "ptx.cuh", "kernels.cuh"], (2, 3)),
+    ("dx", ["ts_gemm.cu", "ptx.cuh", "kernels.cuh"], (3, 4)),
+    ("dw", ["dw_gemm.cu", "ptx.cuh", "kernels.cuh"], (4, 5)),
 ]
 
 
