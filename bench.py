@@ -123,14 +123,21 @@ class ClockSampler:
                 "power_w_max": max(pw) if pw else None}
 
 
-def dist_setup(n_gpus):
+def dist_setup(n_gpus, backend=None):
+    """Rank, world size and local rank from the torchrun environment; joins the
+    process group when world > 1 (NCCL with a GPU per rank, gloo otherwise)."""
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if world > 1:
         import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        if backend is None:
+            backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+            dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        else:
+            dist.init_process_group(backend)
     elif torch.cuda.is_available():
         torch.cuda.set_device(0)
     return rank, world, local
@@ -143,12 +150,21 @@ def barrier(world):
 
 
 def max_over_ranks(x: float, world: int) -> float:
+    """The maximum of x over all ranks (the slowest rank's time)."""
     if world == 1:
         return x
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def whole_job(units_per_rank: float, world: int, max_ms: float, steps: int):
+    """Weak scaling: every rank processes units_per_rank per step; the job's rate
+    is all ranks' units over the slowest rank's time (ms for `steps` steps)."""
+    ms_per_step = max_ms / steps
+    return world * units_per_rank / (ms_per_step * 1e-3), ms_per_step
 
 
 # ------------------------------------------------------------------ the step
@@ -480,8 +496,8 @@ def main():
     with ClockSampler(local) as clk:
         total_ms, per = time_prefill(p, args.steps, args.warmup, world)
     total_ms = max_over_ranks(total_ms, world)
-    ms = total_ms / args.steps
-    value = world * p.flops / (ms * 1e-3) / 1e12
+    rate, ms = whole_job(p.flops, world, total_ms, args.steps)
+    value = rate / 1e12
 
     pk, pk_kind = peaks()
     gemm_flops = 2.0 * p.m * p.n * p.k
@@ -505,7 +521,12 @@ def main():
             "peak_kind": f"{pk_kind} bf16 dense (burst)",
             "algorithmic_per_launch": gemm_flops}
 
-    e2e_ms, h2d, d2h = time_e2e(p, max(5, args.steps // 10), 2)
+    e2e_steps = max(5, args.steps // 10)
+    barrier(world)
+    e2e_ms, h2d, d2h = time_e2e(p, e2e_steps, 2)
+    barrier(world)
+    e2e_rate, e2e_ms = whole_job(p.flops, world, max_over_ranks(e2e_ms * e2e_steps, world),
+                                 e2e_steps)
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
@@ -518,7 +539,7 @@ def main():
                    "replicas": world},
         "roofline": roof,
         "kernels": kinfo,
-        "e2e": {"value": round(world * p.flops / (e2e_ms * 1e-3) / 1e12, 2), "unit": "TFLOP/s",
+        "e2e": {"value": round(e2e_rate / 1e12, 2), "unit": "TFLOP/s",
                 "ms_per_step": round(e2e_ms, 3), "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": len(KERNELS) * args.steps,
