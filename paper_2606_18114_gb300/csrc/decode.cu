@@ -185,8 +185,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
   constexpr int kConsumers = DecodeCfg<kTwoTiles>::kConsumers;
   constexpr int kSplit = DecodeCfg<kTwoTiles>::kSplit;
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* head = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* head = align_shared<1024>(smem_raw);
   const int ub_bytes = b.ubuf_bytes;       // one unit-scale buffer (0: none in this launch)
   float* red = reinterpret_cast<float*>(head + kHeadBytes);  // [2][kRowWarps][32][8]
   uint8_t* ubuf = head + kHeadBytes + kRedBytes;             // two unit-scale buffers

@@ -20,6 +20,15 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// The first A-aligned byte of a dynamic shared-memory array, as an offset from
+// the array itself so that the compiler keeps the shared address space (shared
+// loads rather than generic ones) for every pointer derived from it.
+template <int A>
+__device__ __forceinline__ uint8_t* align_shared(uint8_t* raw) {
+  const uint32_t a = smem_u32(raw);
+  return raw + ((A - (a & (A - 1))) & (A - 1));
+}
+
 __device__ __forceinline__ uint64_t globaltimer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));

@@ -110,8 +110,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   extern __shared__ uint8_t smem_raw[];
   __shared__ int64_t stage_of[kStages];  // local stage held by each slot; -1: end of stream
   __shared__ int mat_of[kStages];        // its matrix
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 127) &
-                                             ~static_cast<uintptr_t>(127));
+  uint8_t* smem = align_shared<128>(smem_raw);
   const uint32_t ring = smem_u32(smem);
   const uint32_t bars = ring + kStages * kStageBytes;
   auto full_bar = [&](int s) { return bars + 8 * s; };

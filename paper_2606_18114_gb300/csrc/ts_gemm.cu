@@ -106,8 +106,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   using L = TsLayout<MODE, BN>;
   constexpr int kSmem = L::kSmem, kAS = L::kAStages, kAcc = L::kAcc;
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* smem = align_shared<1024>(smem_raw);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int64_t rows = MODE == kTsFwd ? args.wn : args.wk;
