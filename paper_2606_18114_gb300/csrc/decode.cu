@@ -48,6 +48,7 @@
 
 #include <algorithm>
 #include <atomic>
+#include <type_traits>
 
 #include "kernels.cuh"
 #include "ptx.cuh"
@@ -424,92 +425,101 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
 #pragma unroll
         for (int i = 0; i < 4; ++i) acc[r][i] = acc1[r][i] = 0.f;
     }
+    // Segments that lie inside k (all but a ragged last one) run without the
+    // per-lane range guards.
+    auto chunks = [&](auto guard) {
+      constexpr bool kGuard = decltype(guard)::value;
 #pragma unroll
-    for (int cc = 0; cc < kChunks / kSplit; ++cc) {
-      const int c = kh * (kChunks / kSplit) + cc;
-      const int64_t kc = static_cast<int64_t>(si.seg) * kSegK + 128 * c;  // chunk start
-      if (kc >= k) break;
-      const bool kin = kc + 32 * t + 32 <= k;  // this lane's 32 offsets lie inside k
-      // The codes box is 128-byte swizzled: 16-byte chunk j of row r sits at chunk
-      // j ^ (r % 8); every row of this lane has r % 8 = g.
-      const int co = (((2 * c + (t >> 1)) ^ g) << 4) + (t & 1) * 8;
-      uint2 w[kTiles][2];
-#pragma unroll
-      for (int r = 0; r < kTiles; ++r) {
-        const uint8_t* cw = cbase + (rl + 16 * r) * (kSegK / 4) + co;
-        w[r][0] = *reinterpret_cast<const uint2*>(cw);
-        w[r][1] = *reinterpret_cast<const uint2*>(cw + 8 * (kSegK / 4));
-      }
-      // past k (a lane of a half chunk) the slot holds no x
-      uint4 xv[4], yv[4];
-      const int xo = (128 * c + 32 * t) * 2;
-      const uint4* xa = reinterpret_cast<const uint4*>(xs + tok0 * kXRowBytes + xo);
-      const uint4* xb = reinterpret_cast<const uint4*>(xs + tok1 * kXRowBytes + xo);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        xv[i] = kin ? xa[i] : make_uint4(0, 0, 0, 0);
-        if (kTwoTiles) yv[i] = kin ? xb[i] : make_uint4(0, 0, 0, 0);
-      }
-      const uint32_t* xr = reinterpret_cast<const uint32_t*>(xv);
-      const uint32_t* yr = reinterpret_cast<const uint32_t*>(yv);
-      if (log2g >= 7) {
-        // exact path: the chunk lies in one group; its products are accumulated
-        // from zero and folded in with the fp32 factor s/2 of that group
-        float p[kTiles][4], p1[kTiles][4];
-#pragma unroll
-        for (int kb = 0; kb < 8; ++kb) {
-          const int j = 2 * (kb & 3);
-#pragma unroll
-          for (int r = 0; r < kTiles; ++r) {
-            const uint32_t u0 = kb < 4 ? w[r][0].x : w[r][0].y;
-            const uint32_t u1 = kb < 4 ? w[r][1].x : w[r][1].y;
-            const uint32_t a0 = pair_bits(u0, j, mul[j]), a1 = pair_bits(u1, j, mul[j]);
-            const uint32_t a2 = pair_bits(u0, j + 1, mul[j + 1]);
-            const uint32_t a3 = pair_bits(u1, j + 1, mul[j + 1]);
-            if (kb == 0) {
-              mma16816_zc(p[r], a0, a1, a2, a3, xr[0], xr[1]);
-              if (kTwoTiles) mma16816_zc(p1[r], a0, a1, a2, a3, yr[0], yr[1]);
-            } else {
-              mma16816(p[r], a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
-              if (kTwoTiles) mma16816(p1[r], a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
-            }
-          }
-        }
-        // C slots 0, 1: row rl + 16r, slots 2, 3: row rl + 16r + 8
-        const int q = static_cast<int>(kc >> log2g) - sq0;
+      for (int cc = 0; cc < kChunks / kSplit; ++cc) {
+        const int c = kh * (kChunks / kSplit) + cc;
+        const int64_t kc = static_cast<int64_t>(si.seg) * kSegK + 128 * c;  // chunk start
+        if (kGuard && kc >= k) break;
+        const bool kin = !kGuard || kc + 32 * t + 32 <= k;  // this lane's 32 offsets lie inside k
+        // The codes box is 128-byte swizzled: 16-byte chunk j of row r sits at chunk
+        // j ^ (r % 8); every row of this lane has r % 8 = g.
+        const int co = (((2 * c + (t >> 1)) ^ g) << 4) + (t & 1) * 8;
+        uint2 w[kTiles][2];
 #pragma unroll
         for (int r = 0; r < kTiles; ++r) {
-          const float h0 = 0.5f * sp[(rl + 16 * r) * sstride + q];
-          const float h1 = 0.5f * sp[(rl + 16 * r + 8) * sstride + q];
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            acc[r][i] = fmaf(i < 2 ? h0 : h1, p[r][i], acc[r][i]);
-            if (kTwoTiles) acc1[r][i] = fmaf(i < 2 ? h0 : h1, p1[r][i], acc1[r][i]);
-          }
+          const uint8_t* cw = cbase + (rl + 16 * r) * (kSegK / 4) + co;
+          w[r][0] = *reinterpret_cast<const uint2*>(cw);
+          w[r][1] = *reinterpret_cast<const uint2*>(cw + 8 * (kSegK / 4));
         }
-      } else {
-        // g = 32 or 64: lane t's offsets 32t .. 32t + 31 of a chunk lie in one
-        // group, whose bf16(s)/2 multiplies the expanded pairs
-        const int q = static_cast<int>((kc + 32 * t) >> log2g) - sq0;
+        // past k (a lane of a half chunk) the slot holds no x
+        uint4 xv[4], yv[4];
+        const int xo = (128 * c + 32 * t) * 2;
+        const uint4* xa = reinterpret_cast<const uint4*>(xs + tok0 * kXRowBytes + xo);
+        const uint4* xb = reinterpret_cast<const uint4*>(xs + tok1 * kXRowBytes + xo);
 #pragma unroll
-        for (int r = 0; r < kTiles; ++r) {
-          const uint32_t hs0 = kin ? half_scale_bf16x2(sp[(rl + 16 * r) * sstride + q]) : 0u;
-          const uint32_t hs1 = kin ? half_scale_bf16x2(sp[(rl + 16 * r + 8) * sstride + q]) : 0u;
+        for (int i = 0; i < 4; ++i) {
+          xv[i] = kin ? xa[i] : make_uint4(0, 0, 0, 0);
+          if (kTwoTiles) yv[i] = kin ? xb[i] : make_uint4(0, 0, 0, 0);
+        }
+        const uint32_t* xr = reinterpret_cast<const uint32_t*>(xv);
+        const uint32_t* yr = reinterpret_cast<const uint32_t*>(yv);
+        if (log2g >= 7) {
+          // exact path: the chunk lies in one group; its products are accumulated
+          // from zero and folded in with the fp32 factor s/2 of that group
+          float p[kTiles][4], p1[kTiles][4];
 #pragma unroll
           for (int kb = 0; kb < 8; ++kb) {
             const int j = 2 * (kb & 3);
-            const uint32_t u0 = kb < 4 ? w[r][0].x : w[r][0].y;
-            const uint32_t u1 = kb < 4 ? w[r][1].x : w[r][1].y;
-            const uint32_t a0 = bmul2(pair_bits(u0, j, mul[j]), hs0);
-            const uint32_t a1 = bmul2(pair_bits(u1, j, mul[j]), hs1);
-            const uint32_t a2 = bmul2(pair_bits(u0, j + 1, mul[j + 1]), hs0);
-            const uint32_t a3 = bmul2(pair_bits(u1, j + 1, mul[j + 1]), hs1);
-            mma16816(acc[r], a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
-            if (kTwoTiles) mma16816(acc1[r], a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
+#pragma unroll
+            for (int r = 0; r < kTiles; ++r) {
+              const uint32_t u0 = kb < 4 ? w[r][0].x : w[r][0].y;
+              const uint32_t u1 = kb < 4 ? w[r][1].x : w[r][1].y;
+              const uint32_t a0 = pair_bits(u0, j, mul[j]), a1 = pair_bits(u1, j, mul[j]);
+              const uint32_t a2 = pair_bits(u0, j + 1, mul[j + 1]);
+              const uint32_t a3 = pair_bits(u1, j + 1, mul[j + 1]);
+              if (kb == 0) {
+                mma16816_zc(p[r], a0, a1, a2, a3, xr[0], xr[1]);
+                if (kTwoTiles) mma16816_zc(p1[r], a0, a1, a2, a3, yr[0], yr[1]);
+              } else {
+                mma16816(p[r], a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
+                if (kTwoTiles) mma16816(p1[r], a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
+              }
+            }
+          }
+          // C slots 0, 1: row rl + 16r, slots 2, 3: row rl + 16r + 8
+          const int q = static_cast<int>(kc >> log2g) - sq0;
+#pragma unroll
+          for (int r = 0; r < kTiles; ++r) {
+            const float h0 = 0.5f * sp[(rl + 16 * r) * sstride + q];
+            const float h1 = 0.5f * sp[(rl + 16 * r + 8) * sstride + q];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              acc[r][i] = fmaf(i < 2 ? h0 : h1, p[r][i], acc[r][i]);
+              if (kTwoTiles) acc1[r][i] = fmaf(i < 2 ? h0 : h1, p1[r][i], acc1[r][i]);
+            }
+          }
+        } else {
+          // g = 32 or 64: lane t's offsets 32t .. 32t + 31 of a chunk lie in one
+          // group, whose bf16(s)/2 multiplies the expanded pairs
+          const int q = static_cast<int>((kc + 32 * t) >> log2g) - sq0;
+#pragma unroll
+          for (int r = 0; r < kTiles; ++r) {
+            const uint32_t hs0 = kin ? half_scale_bf16x2(sp[(rl + 16 * r) * sstride + q]) : 0u;
+            const uint32_t hs1 = kin ? half_scale_bf16x2(sp[(rl + 16 * r + 8) * sstride + q]) : 0u;
+#pragma unroll
+            for (int kb = 0; kb < 8; ++kb) {
+              const int j = 2 * (kb & 3);
+              const uint32_t u0 = kb < 4 ? w[r][0].x : w[r][0].y;
+              const uint32_t u1 = kb < 4 ? w[r][1].x : w[r][1].y;
+              const uint32_t a0 = bmul2(pair_bits(u0, j, mul[j]), hs0);
+              const uint32_t a1 = bmul2(pair_bits(u1, j, mul[j]), hs1);
+              const uint32_t a2 = bmul2(pair_bits(u0, j + 1, mul[j + 1]), hs0);
+              const uint32_t a3 = bmul2(pair_bits(u1, j + 1, mul[j + 1]), hs1);
+              mma16816(acc[r], a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
+              if (kTwoTiles) mma16816(acc1[r], a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
+            }
           }
         }
       }
-    }
+    };
+    if (!kTwoTiles && static_cast<int64_t>(si.seg + 1) * kSegK <= k)
+      chunks(std::integral_constant<bool, false>{});  // (two n-tiles: no register room)
+    else
+      chunks(std::integral_constant<bool, true>{});
     __syncwarp();
     if (lane == 0) {
       mbar_arrive(empty_bar(slot));
