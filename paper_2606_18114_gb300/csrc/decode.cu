@@ -110,7 +110,9 @@ __device__ __forceinline__ uint32_t bmul2(uint32_t a, uint32_t b) {
 // 30-31 (exact, the fields are 16 bits apart). mul is a register whose value the
 // compiler does not see, so the move runs as an integer multiply on the FMA pipe
 // instead of a shift on the ALU pipe, which the mask already loads.
+// Pair 7 already sits at bits 14-15 and 30-31: the mask alone.
 __device__ __forceinline__ uint32_t pair_bits(uint32_t w, int j, uint32_t mul) {
+  if (j == 7) return w & 0xC000C000u;
   return (w & (0x00030003u << (2 * j))) * mul;
 }
 
