@@ -142,6 +142,22 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
                         int32_t accumulate_dw, void* stream);
 
 /*
+ * tq_linear_bwd_noalloc — tq_linear_bwd on the faster transposed-codes dX path
+ * without a caller-provided codes_t: the codes are transposed (tq_codes_transpose)
+ * into a 16 MB scratch array inside the library (a file-scope device array; no
+ * allocation at any time), then the product runs as tq_linear_bwd with it. Same
+ * arguments and results as tq_linear_bwd with codes_t = NULL.
+ *   Returns TQ_ERR_UNSUPPORTED when the transposed codes (k * 4 * ceil(n/64)
+ *   words) exceed the scratch; pass codes_t to tq_linear_bwd then.
+ *   The scratch is one per device: calls on one device must not overlap in time
+ *   (issue them on one stream).
+ */
+TQ_API tq_status tq_linear_bwd_noalloc(const void* dy, const void* x, int64_t m, int64_t n,
+                                       int64_t k, const uint32_t* codes, const float* scales,
+                                       int32_t g, void* dx, int32_t dx_dtype, float* dw,
+                                       int32_t accumulate_dw, void* stream);
+
+/*
  * tq_codes_transpose — the packed codes of W^T, a re-layout of tq_quantize's codes
  * (no arithmetic of the method) that the STE dX product streams along its
  * reduction (n):

@@ -11,6 +11,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <atomic>
 #include <mutex>
 #include <unordered_map>
 
@@ -412,11 +413,10 @@ TQ_API tq_status tq_codes_transpose(const uint32_t* codes, int64_t n, int64_t k,
   return e == cudaSuccess ? TQ_OK : cuda_fail(e, "transpose launch");
 }
 
-TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t n, int64_t k,
-                               const uint32_t* codes, const uint32_t* codes_t,
-                               const float* scales, int32_t g, void* dx, int32_t dx_dtype,
-                               float* dw, int32_t accumulate_dw, void* stream) {
-  g_err[0] = 0;
+// Arguments of the backward, checked before anything is enqueued.
+tq_status check_bwd_args(const void* dy, const void* x, int64_t m, int64_t n, int64_t k,
+                         const uint32_t* codes, const uint32_t* codes_t, const float* scales,
+                         int32_t g, const void* dx, int32_t dx_dtype, const float* dw) {
   TQ_TRY(check_linear_shape(m, n, k, g));
   if (n % 8 != 0)
     return fail(TQ_ERR_UNSUPPORTED, "n=%lld: the backward kernels need n %% 8 == 0", (long long)n);
@@ -441,6 +441,17 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
       TQ_TRY(check_ptr(x, "x"));
     }
   }
+  return TQ_OK;
+}
+
+TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t n, int64_t k,
+                               const uint32_t* codes, const uint32_t* codes_t,
+                               const float* scales, int32_t g, void* dx, int32_t dx_dtype,
+                               float* dw, int32_t accumulate_dw, void* stream) {
+  g_err[0] = 0;
+  TQ_TRY(check_bwd_args(dy, x, m, n, k, codes, codes_t, scales, g, dx, dx_dtype, dw));
+  const bool want_dx = dx != nullptr && m > 0 && k > 0;
+  const bool want_dw = dw != nullptr && n > 0 && k > 0;
   if (!want_dx && !want_dw) return TQ_OK;
   const DeviceInfo* dev = nullptr;
   TQ_TRY(device_info(&dev));
@@ -528,3 +539,55 @@ TQ_API tq_status tq_device_status(void* stream) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------- no-alloc backward
+// Scratch for the transposed codes of tq_linear_bwd_noalloc: a file-scope device
+// array, so the caller allocates nothing. One per device; calls that use it must
+// not overlap in time on one device (keep them on one stream).
+constexpr int64_t kNoAllocWords = int64_t(4) << 20;  // 16 MB of uint32 words
+static __device__ __align__(256) uint32_t g_codes_t_scratch[kNoAllocWords];
+
+namespace {
+tq_status noalloc_scratch(uint32_t** out) {
+  static std::atomic<uintptr_t> base[kMaxDevices];
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return fail(TQ_ERR_UNSUPPORTED, "device %d", dev);
+  uintptr_t p = base[dev].load(std::memory_order_acquire);
+  if (p == 0) {
+    void* a = nullptr;
+    if ((e = cudaGetSymbolAddress(&a, g_codes_t_scratch)) != cudaSuccess)
+      return cuda_fail(e, "cudaGetSymbolAddress");
+    p = reinterpret_cast<uintptr_t>(a);
+    base[dev].store(p, std::memory_order_release);
+  }
+  *out = reinterpret_cast<uint32_t*>(p);
+  return TQ_OK;
+}
+}  // namespace
+
+TQ_API tq_status tq_linear_bwd_noalloc(const void* dy, const void* x, int64_t m, int64_t n,
+                                       int64_t k, const uint32_t* codes, const float* scales,
+                                       int32_t g, void* dx, int32_t dx_dtype, float* dw,
+                                       int32_t accumulate_dw, void* stream) {
+  g_err[0] = 0;
+  const bool want_dx = dx != nullptr && m > 0 && k > 0 && n > 0;
+  if (!want_dx)  // nothing to transpose: exactly tq_linear_bwd
+    return tq_linear_bwd(dy, x, m, n, k, codes, nullptr, scales, g, dx, dx_dtype, dw,
+                         accumulate_dw, stream);
+  TQ_TRY(check_bwd_args(dy, x, m, n, k, codes, nullptr, scales, g, dx, dx_dtype, dw));
+  const int64_t ldt = 4 * ((n + 63) / 64);
+  if (k > kNoAllocWords / ldt)
+    return fail(TQ_ERR_UNSUPPORTED,
+                "transposed codes of n=%lld k=%lld need %lld words, scratch holds %lld; pass "
+                "codes_t to tq_linear_bwd instead",
+                (long long)n, (long long)k, (long long)(ldt * k), (long long)kNoAllocWords);
+  uint32_t* scratch = nullptr;
+  TQ_TRY(noalloc_scratch(&scratch));
+  const cudaError_t e =
+      tq::launch_transpose_codes(codes, n, k, scratch, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "transpose launch");
+  return tq_linear_bwd(dy, x, m, n, k, codes, scratch, scales, g, dx, dx_dtype, dw,
+                       accumulate_dw, stream);
+}

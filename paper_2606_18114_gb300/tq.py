@@ -20,6 +20,7 @@ __all__ = [
     "quant_batch",
     "linear_fwd",
     "linear_bwd",
+    "linear_bwd_noalloc",
     "codes_transpose",
     "linear_fwd_batched",
     "fwd_batch",
@@ -36,8 +37,8 @@ STATUS = {0: "TQ_OK", 1: "TQ_ERR_INVALID_ARG", 2: "TQ_ERR_UNSUPPORTED", 3: "TQ_E
           4: "TQ_ERR_TIMEOUT"}
 # Every symbol include/tq.h declares.
 EXPORTS = ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
-           "tq_codes_transpose", "tq_linear_fwd_batched", "tq_device_status", "tq_last_error",
-           "tq_version")
+           "tq_linear_bwd_noalloc", "tq_codes_transpose", "tq_linear_fwd_batched",
+           "tq_device_status", "tq_last_error", "tq_version")
 
 _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtq.so")
 _lib = None
@@ -87,11 +88,14 @@ def load(path: Optional[str] = None):
     lib.tq_quantize_batched.argtypes = [ctypes.POINTER(QuantDesc), i32, i32, vp]
     lib.tq_linear_fwd.argtypes = [vp, i64, i64, vp, vp, i64, i32, vp, i32, vp]
     lib.tq_linear_bwd.argtypes = [vp, vp, i64, i64, i64, vp, vp, vp, i32, vp, i32, vp, i32, vp]
+    lib.tq_linear_bwd_noalloc.argtypes = [vp, vp, i64, i64, i64, vp, vp, i32, vp, i32, vp, i32,
+                                          vp]
     lib.tq_codes_transpose.argtypes = [vp, i64, i64, vp, vp]
     lib.tq_linear_fwd_batched.argtypes = [ctypes.POINTER(FwdDesc), i32, i64, vp]
     lib.tq_device_status.argtypes = [vp]
     for name in ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
-                 "tq_codes_transpose", "tq_linear_fwd_batched", "tq_device_status"):
+                 "tq_linear_bwd_noalloc", "tq_codes_transpose", "tq_linear_fwd_batched",
+                 "tq_device_status"):
         getattr(lib, name).restype = ctypes.c_int
     lib.tq_last_error.restype = ctypes.c_char_p
     lib.tq_last_error.argtypes = []
@@ -218,6 +222,28 @@ def linear_bwd(dy: torch.Tensor, x: Optional[torch.Tensor], codes: torch.Tensor,
                                 _ptr(scales), g,
                                 _ptr(dx), _out_code(dx.dtype) if dx is not None else OUT_F32,
                                 _ptr(dw), int(accumulate_dw), _stream(stream)))
+    return dx, dw
+
+
+def linear_bwd_noalloc(dy: torch.Tensor, x: Optional[torch.Tensor], codes: torch.Tensor,
+                       scales: torch.Tensor, k: int, g: int, want_dx: bool = True,
+                       want_dw: bool = True, dx_dtype=torch.float32,
+                       dx: Optional[torch.Tensor] = None, dw: Optional[torch.Tensor] = None,
+                       accumulate_dw: bool = False, stream=None):
+    """``linear_bwd`` on the transposed-codes dX path with the library's own
+    scratch for the transposed codes (nothing allocated for them)."""
+    m, n = dy.shape
+    if want_dx and dx is None:
+        dx = torch.empty((m, k), dtype=dx_dtype, device=dy.device)
+    if want_dw and dw is None:
+        dw = torch.empty((n, k), dtype=torch.float32, device=dy.device)
+    if not want_dx:
+        dx = None
+    if not want_dw:
+        dw = None
+    _check(load().tq_linear_bwd_noalloc(_ptr(dy), _ptr(x), m, n, k, _ptr(codes), _ptr(scales), g,
+                                        _ptr(dx), _out_code(dx.dtype) if dx is not None else OUT_F32,
+                                        _ptr(dw), int(accumulate_dw), _stream(stream)))
     return dx, dw
 
 
