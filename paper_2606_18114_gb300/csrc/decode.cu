@@ -386,6 +386,21 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
   const int tok0 = g < m ? g : m - 1;  // tokens past m read token m - 1
   const int tok1 = g + 8 < m ? g + 8 : m - 1;
   const int rl = 32 * wr + g;          // row of tile 0 for C slots 0, 1 (+8: slots 2, 3)
+  // Byte offsets inside a slot that do not change from segment to segment: the
+  // codes of this lane's rows for each of its chunks (the 128-byte swizzle moves
+  // 16-byte chunk j of row r to j ^ (r % 8), and every row of this lane has
+  // r % 8 = g), and its x fragments.
+  constexpr int kMine = kChunks / kSplit;  // chunks of a segment this warp takes
+  auto code_at = [&](int c) { return rl * (kSegK / 4) + (((2 * c + (t >> 1)) ^ g) << 4) + (t & 1) * 8; };
+  auto x_at = [&](int tok, int c) { return tok * kXRowBytes + (128 * c + 32 * t) * 2; };
+  // kept in registers up to 8 tokens; recomputed per chunk with two n-tiles,
+  // whose accumulators need the registers
+  int code_off[kMine], x0_off[kMine];
+#pragma unroll
+  for (int cc = 0; cc < kMine; ++cc) {
+    code_off[cc] = code_at(kh * kMine + cc);
+    x0_off[cc] = x_at(tok0, kh * kMine + cc);
+  }
   int units_r = 0;                     // units whose partial sums were handed over
 
   int slot = 0;
@@ -421,6 +436,17 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
       }
     }
     const uint8_t* xs = cbase + kCodeBytes + scale_bytes;  // x [m tokens][kSegK]
+    // this lane's scale rows: tile r, C slots 0-1 (h = 0) and 2-3 (h = 1)
+    const float* srow[kTiles][2];
+#pragma unroll
+    for (int r = 0; r < kTiles; ++r)
+#pragma unroll
+      for (int h = 0; h < 2; ++h) srow[r][h] = sp + (rl + 16 * r + 8 * h) * sstride - sq0;
+    // scale of tile r, C-slot half h and group q (with two n-tiles recomputed
+    // instead of held in registers)
+    auto scale_at = [&](int r, int h, int q) -> float {
+      return kTwoTiles ? sp[(rl + 16 * r + 8 * h) * sstride + q - sq0] : srow[r][h][q];
+    };
     if (si.seg == 0) {
 #pragma unroll
       for (int r = 0; r < kTiles; ++r)
@@ -432,26 +458,22 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     auto chunks = [&](auto guard) {
       constexpr bool kGuard = decltype(guard)::value;
 #pragma unroll
-      for (int cc = 0; cc < kChunks / kSplit; ++cc) {
-        const int c = kh * (kChunks / kSplit) + cc;
+      for (int cc = 0; cc < kMine; ++cc) {
+        const int c = kh * kMine + cc;
         const int64_t kc = static_cast<int64_t>(si.seg) * kSegK + 128 * c;  // chunk start
         if (kGuard && kc >= k) break;
         const bool kin = !kGuard || kc + 32 * t + 32 <= k;  // this lane's 32 offsets lie inside k
-        // The codes box is 128-byte swizzled: 16-byte chunk j of row r sits at chunk
-        // j ^ (r % 8); every row of this lane has r % 8 = g.
-        const int co = (((2 * c + (t >> 1)) ^ g) << 4) + (t & 1) * 8;
         uint2 w[kTiles][2];
 #pragma unroll
         for (int r = 0; r < kTiles; ++r) {
-          const uint8_t* cw = cbase + (rl + 16 * r) * (kSegK / 4) + co;
+          const uint8_t* cw = cbase + (kTwoTiles ? code_at(c) : code_off[cc]) + r * 16 * (kSegK / 4);
           w[r][0] = *reinterpret_cast<const uint2*>(cw);
           w[r][1] = *reinterpret_cast<const uint2*>(cw + 8 * (kSegK / 4));
         }
         // past k (a lane of a half chunk) the slot holds no x
         uint4 xv[4], yv[4];
-        const int xo = (128 * c + 32 * t) * 2;
-        const uint4* xa = reinterpret_cast<const uint4*>(xs + tok0 * kXRowBytes + xo);
-        const uint4* xb = reinterpret_cast<const uint4*>(xs + tok1 * kXRowBytes + xo);
+        const uint4* xa = reinterpret_cast<const uint4*>(xs + (kTwoTiles ? x_at(tok0, c) : x0_off[cc]));
+        const uint4* xb = reinterpret_cast<const uint4*>(xs + x_at(tok1, c));
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           xv[i] = kin ? xa[i] : make_uint4(0, 0, 0, 0);
@@ -483,11 +505,11 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
             }
           }
           // C slots 0, 1: row rl + 16r, slots 2, 3: row rl + 16r + 8
-          const int q = static_cast<int>(kc >> log2g) - sq0;
+          const int q = static_cast<int>(kc >> log2g);
 #pragma unroll
           for (int r = 0; r < kTiles; ++r) {
-            const float h0 = 0.5f * sp[(rl + 16 * r) * sstride + q];
-            const float h1 = 0.5f * sp[(rl + 16 * r + 8) * sstride + q];
+            const float h0 = 0.5f * scale_at(r, 0, q);
+            const float h1 = 0.5f * scale_at(r, 1, q);
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
               acc[r][i] = fmaf(i < 2 ? h0 : h1, p[r][i], acc[r][i]);
@@ -497,11 +519,11 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
         } else {
           // g = 32 or 64: lane t's offsets 32t .. 32t + 31 of a chunk lie in one
           // group, whose bf16(s)/2 multiplies the expanded pairs
-          const int q = static_cast<int>((kc + 32 * t) >> log2g) - sq0;
+          const int q = static_cast<int>((kc + 32 * t) >> log2g);
 #pragma unroll
           for (int r = 0; r < kTiles; ++r) {
-            const uint32_t hs0 = kin ? half_scale_bf16x2(sp[(rl + 16 * r) * sstride + q]) : 0u;
-            const uint32_t hs1 = kin ? half_scale_bf16x2(sp[(rl + 16 * r + 8) * sstride + q]) : 0u;
+            const uint32_t hs0 = kin ? half_scale_bf16x2(scale_at(r, 0, q)) : 0u;
+            const uint32_t hs1 = kin ? half_scale_bf16x2(scale_at(r, 1, q)) : 0u;
 #pragma unroll
             for (int kb = 0; kb < 8; ++kb) {
               const int j = 2 * (kb & 3);
