@@ -40,8 +40,14 @@
 // Expansion: pair j of a code word -> bf16x2 (2c, 2c) by ((w << (14 - 2j)) &
 // 0xC000C000) (layout of include/tq.h). For g >= 128 a chunk lies in one group:
 // each group's products are accumulated from zero and folded into the output
-// with the exact fp32 factor s/2. For g <= 64 the groups of a chunk meet inside
-// one MMA, so the expansion multiplies by bf16(s)/2 as the prefill kernels do.
+// with the exact fp32 scale s, the sums halved (exactly) at the store. For g <= 64
+// the groups of a chunk meet inside one MMA, so the expansion multiplies by
+// bf16(s)/2 as the prefill kernels do.
+//
+// A consumer warp reads a unit's descriptor once, at its first segment, and takes
+// every per-matrix decision there (scale addressing, exact or bf16 scaling, which
+// segments need range guards); per segment it runs one wait, its chunks and one
+// arrival.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -401,66 +407,62 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     code_off[cc] = code_at(kh * kMine + cc);
     x0_off[cc] = x_at(tok0, kh * kMine + cc);
   }
-  int units_r = 0;                     // units whose partial sums were handed over
-
+  int units_r = 0;  // units whose partial sums were handed over
+  int units_u = 0;  // units whose scales came through the unit buffers
   int slot = 0;
   uint32_t parity = 0;
-  int units_u = 0;
   for (;;) {
+    // The first segment of a unit carries the unit's descriptor: everything that
+    // depends on the matrix is decided here once, so that per segment a warp runs
+    // one wait, its chunks and one arrival.
     if (!warp_wait(full_bar(slot), parity, status)) return;
     const SegInfo si = info[slot];
     if (si.mat < 0) break;
-    const int64_t k = si.k;
+    const int k = si.k;
     const int log2g = si.log2g;
     const int mode = si.mode & 0xff;
-    const int g0 = (si.seg * kSegK) >> log2g;  // first group of the segment
-    const uint8_t* cbase = smem + slot * slot_bytes;
-    // scale of unit row r and group q: sp[r * sstride + q - sq0]
-    const float* sp;
-    int sstride, sq0;
     const bool unit_scales = mode == kDecodeScaleUnit;
+    const int nfull = k / kSegK;  // segments that lie inside k
+    const int nseg = (k + kSegK - 1) / kSegK;
+    // Scale of unit row r and group q: area[r * sstride + q - sq0], the area being
+    // the unit buffer (sq0 = 0) or the segment's slot (sq0 = its first stored group).
+    const int sstride = unit_scales ? (k >> log2g)
+                        : mode == kDecodeScale16 ? decode_scale_box(log2g)
+                                                 : (log2g >= 9 ? 1 : kSegK >> log2g);
+    const float* ubase = nullptr;
     if (unit_scales) {
       const int ub = units_u & 1;
-      if (si.seg == 0 && !warp_wait(sfull_bar(ub), (units_u >> 1) & 1, status)) return;
-      sp = reinterpret_cast<const float*>(ubuf + ub * ub_bytes);
-      sstride = static_cast<int>(k >> log2g);
-      sq0 = 0;
-    } else {
-      sp = reinterpret_cast<const float*>(cbase + kCodeBytes);
-      if (mode == kDecodeScale16) {
-        sstride = decode_scale_box(log2g);
-        sq0 = g0 - g0 % sstride;
-      } else {
-        sstride = log2g >= 9 ? 1 : kSegK >> log2g;
-        sq0 = g0;
-      }
+      if (!warp_wait(sfull_bar(ub), (units_u >> 1) & 1, status)) return;
+      ubase = reinterpret_cast<const float*>(ubuf + ub * ub_bytes);
     }
-    const uint8_t* xs = cbase + kCodeBytes + scale_bytes;  // x [m tokens][kSegK]
-    // this lane's scale rows: tile r, C slots 0-1 (h = 0) and 2-3 (h = 1)
-    const float* srow[kTiles][2];
+    const int srl = rl * sstride;  // this lane's row of tile 0, C slots 0-1
+    const int s8 = 8 * sstride;    // + 8 rows: C slots 2-3; + 16 rows: the next tile
 #pragma unroll
     for (int r = 0; r < kTiles; ++r)
 #pragma unroll
-      for (int h = 0; h < 2; ++h) srow[r][h] = sp + (rl + 16 * r + 8 * h) * sstride - sq0;
-    // scale of tile r, C-slot half h and group q (with two n-tiles recomputed
-    // instead of held in registers)
-    auto scale_at = [&](int r, int h, int q) -> float {
-      return kTwoTiles ? sp[(rl + 16 * r + 8 * h) * sstride + q - sq0] : srow[r][h][q];
-    };
-    if (si.seg == 0) {
-#pragma unroll
-      for (int r = 0; r < kTiles; ++r)
-#pragma unroll
-        for (int i = 0; i < 4; ++i) acc[r][i] = acc1[r][i] = 0.f;
-    }
-    // Segments that lie inside k (all but a ragged last one) run without the
-    // per-lane range guards.
-    auto chunks = [&](auto guard) {
+      for (int i = 0; i < 4; ++i) acc[r][i] = acc1[r][i] = 0.f;
+
+    // Segment s of the unit: its wait (the first one's was the descriptor's), this
+    // warp's chunks, the release of the slot. kGuard: the segment reaches past k.
+    // kExact (g >= 128): a chunk lies in one group; its products are accumulated
+    // from zero and folded in with the fp32 scale s (the expanded codes are 2c, so
+    // the sums are twice the output, halved exactly at the store). Otherwise
+    // (g = 32, 64) lane t's offsets 32t .. 32t + 31 of a chunk lie in one group,
+    // whose bf16(s)/2 multiplies the expanded pairs.
+    auto segment = [&](int s, auto guard, auto exact) -> bool {
       constexpr bool kGuard = decltype(guard)::value;
+      constexpr bool kExact = decltype(exact)::value;
+      if (s > 0 && !warp_wait(full_bar(slot), parity, status)) return false;
+      const uint8_t* cbase = smem + slot * slot_bytes;
+      const int g0 = (s * kSegK) >> log2g;  // first group of the segment
+      const float* sl = unit_scales ? ubase
+                        : reinterpret_cast<const float*>(cbase + kCodeBytes) -
+                              (mode == kDecodeScale16 ? (g0 & -sstride) : g0);
+      const uint8_t* xs = cbase + kCodeBytes + scale_bytes;  // x [m tokens][kSegK]
 #pragma unroll
       for (int cc = 0; cc < kMine; ++cc) {
         const int c = kh * kMine + cc;
-        const int64_t kc = static_cast<int64_t>(si.seg) * kSegK + 128 * c;  // chunk start
+        const int kc = s * kSegK + 128 * c;  // chunk start
         if (kGuard && kc >= k) break;
         const bool kin = !kGuard || kc + 32 * t + 32 <= k;  // this lane's 32 offsets lie inside k
         uint2 w[kTiles][2];
@@ -481,9 +483,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
         }
         const uint32_t* xr = reinterpret_cast<const uint32_t*>(xv);
         const uint32_t* yr = reinterpret_cast<const uint32_t*>(yv);
-        if (log2g >= 7) {
-          // exact path: the chunk lies in one group; its products are accumulated
-          // from zero and folded in with the fp32 factor s/2 of that group
+        if constexpr (kExact) {
           float p[kTiles][4], p1[kTiles][4];
 #pragma unroll
           for (int kb = 0; kb < 8; ++kb) {
@@ -505,11 +505,11 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
             }
           }
           // C slots 0, 1: row rl + 16r, slots 2, 3: row rl + 16r + 8
-          const int q = static_cast<int>(kc >> log2g);
+          const int q = kc >> log2g;
 #pragma unroll
           for (int r = 0; r < kTiles; ++r) {
-            const float h0 = 0.5f * scale_at(r, 0, q);
-            const float h1 = 0.5f * scale_at(r, 1, q);
+            const float h0 = sl[srl + 2 * r * s8 + q];
+            const float h1 = sl[srl + (2 * r + 1) * s8 + q];
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
               acc[r][i] = fmaf(i < 2 ? h0 : h1, p[r][i], acc[r][i]);
@@ -517,13 +517,11 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
             }
           }
         } else {
-          // g = 32 or 64: lane t's offsets 32t .. 32t + 31 of a chunk lie in one
-          // group, whose bf16(s)/2 multiplies the expanded pairs
-          const int q = static_cast<int>((kc + 32 * t) >> log2g);
+          const int q = (kc + 32 * t) >> log2g;
 #pragma unroll
           for (int r = 0; r < kTiles; ++r) {
-            const uint32_t hs0 = kin ? half_scale_bf16x2(scale_at(r, 0, q)) : 0u;
-            const uint32_t hs1 = kin ? half_scale_bf16x2(scale_at(r, 1, q)) : 0u;
+            const uint32_t hs0 = kin ? half_scale_bf16x2(sl[srl + 2 * r * s8 + q]) : 0u;
+            const uint32_t hs1 = kin ? half_scale_bf16x2(sl[srl + (2 * r + 1) * s8 + q]) : 0u;
 #pragma unroll
             for (int kb = 0; kb < 8; ++kb) {
               const int j = 2 * (kb & 3);
@@ -539,18 +537,35 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
           }
         }
       }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty_bar(slot));
+      if (++slot == stages) {
+        slot = 0;
+        parity ^= 1u;
+      }
+      return true;
     };
-    if (!kTwoTiles && static_cast<int64_t>(si.seg + 1) * kSegK <= k)
-      chunks(std::integral_constant<bool, false>{});  // (two n-tiles: no register room)
+    bool ok = true;
+    auto run = [&](auto exact) {
+      if constexpr (kTwoTiles) {
+        // (two n-tiles: no register room for a second chunk body)
+        for (int s = 0; s < nseg && ok; ++s) ok = segment(s, std::true_type{}, exact);
+      } else {
+        for (int s = 0; s < nfull && ok; ++s) ok = segment(s, std::false_type{}, exact);
+        if (ok && nfull < nseg) ok = segment(nfull, std::true_type{}, exact);
+      }
+    };
+    const bool exact = log2g >= 7;
+    if (exact)
+      run(std::true_type{});
     else
-      chunks(std::integral_constant<bool, true>{});
-    __syncwarp();
-    if (lane == 0) {
-      mbar_arrive(empty_bar(slot));
-      if (unit_scales && si.last) mbar_arrive(sempty_bar(units_u & 1));
+      run(std::false_type{});
+    if (!ok) return;
+    if (unit_scales) {
+      if (lane == 0) mbar_arrive(sempty_bar(units_u & 1));
+      ++units_u;
     }
-    if (unit_scales && si.last) ++units_u;
-    if (si.last && kSplit == 2) {
+    if (kSplit == 2) {
       // the second warp of the slice hands its partial sums to the first through
       // buffer units_r % 2 (bounded waits both ways: "written" and "read")
       const int pb = units_r & 1;
@@ -575,16 +590,17 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
       }
       ++units_r;
     }
-    if (si.last && kh == 0) {
+    if (kh == 0) {
       // C fragment of tile r: rows rl + 16r (slots 0, 1) and + 8 (2, 3), tokens 2t, 2t + 1
       const int64_t n = si.n;
       const bool ybf16 = (si.mode >> 8) != 0;
+      const float post = exact ? 0.5f : 1.f;
       auto store = [&](int token, int64_t row, float v) {
         if (token < m && row < n) {
           if (ybf16)
-            static_cast<__nv_bfloat16*>(si.y)[token * n + row] = __float2bfloat16_rn(v);
+            static_cast<__nv_bfloat16*>(si.y)[token * n + row] = __float2bfloat16_rn(post * v);
           else
-            static_cast<float*>(si.y)[token * n + row] = v;
+            static_cast<float*>(si.y)[token * n + row] = post * v;
         }
       };
 #pragma unroll
@@ -601,10 +617,6 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
           store(8 + 2 * t + 1, rb, acc1[r][3]);
         }
       }
-    }
-    if (++slot == stages) {
-      slot = 0;
-      parity ^= 1u;
     }
   }
 }
