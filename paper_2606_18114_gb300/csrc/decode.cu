@@ -75,10 +75,15 @@ struct DecodeCfg {
   static constexpr int kThreads = (kConsumers + 1) * 32;  // + one producer warp
 };
 constexpr int kRedBytes = 2 * kRowWarps * 32 * kTiles * 4 * 4;  // partial sums, two units
+// (the hand-off area exists only where two warps share a row slice)
+template <bool kTwoTiles>
+__host__ __device__ constexpr int red_bytes() { return kTwoTiles ? 0 : kRedBytes; }
 constexpr int kSegK = kDecodeSegK;               // k per segment (one TMA box of 32 words)
 constexpr int kChunks = kSegK / 128;             // 128-wide chunks per segment
 constexpr int kCodeBytes = kRows * kSegK / 4;    // 32 KB
-constexpr int kXRowBytes = kSegK * 2;            // one token's bf16 slice of the segment
+// x of one token over a segment (1 KB), tokens 1040 bytes apart (= 16 mod 128) so
+// that the two tokens of a quarter-warp read disjoint shared-memory banks.
+constexpr int kXTokBytes = kSegK * 2 + 16;
 constexpr int kMaxStages = 8;
 constexpr int kHeadBytes = 1024;                 // barriers and segment descriptors
 constexpr int kSmemLimit = 227 * 1024;
@@ -87,6 +92,20 @@ constexpr int kSmemLimit = 227 * 1024;
 
 static_assert(kRowWarps == 8, "two m16 row tiles per row warp");
 static_assert(kCodeBytes == 32 * 1024, "codes box");
+
+// Row strides (in floats) of the scale areas. The eight rows a warp reads at once
+// (rows = 0..7 mod 8) fall on distinct banks when the stride in 16-byte units is
+// odd, hence a 16-byte pad on rows of an even number of 16-byte units (one float
+// for the 4-byte mode) where the producer copies rows one by one. A unit's scales
+// arrive in one bulk copy and keep their rows gpr apart (per-row copies into
+// padded rows cost more than the bank conflicts they remove).
+__host__ __device__ constexpr int unit_scale_stride(int gpr) { return gpr; }
+__host__ __device__ constexpr int box_scale_stride(int log2g) {
+  return decode_scale_box(log2g) % 8 == 0 ? decode_scale_box(log2g) + 4 : decode_scale_box(log2g);
+}
+__host__ __device__ constexpr int seg_scale_stride(int log2g) {
+  return (log2g >= 9 ? 1 : kSegK >> log2g) | 1;
+}
 
 // Segment descriptor written by the producer next to the slot's barriers; it
 // carries what the consumers need of the matrix, so they never index the
@@ -197,7 +216,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
   uint8_t* head = align_shared<1024>(smem_raw);
   const int ub_bytes = b.ubuf_bytes;       // one unit-scale buffer (0: none in this launch)
   float* red = reinterpret_cast<float*>(head + kHeadBytes);  // [2][kRowWarps][32][8]
-  uint8_t* ubuf = head + kHeadBytes + kRedBytes;             // two unit-scale buffers
+  uint8_t* ubuf = head + kHeadBytes + red_bytes<kTwoTiles>();  // two unit-scale buffers
   uint8_t* smem = ubuf + 2 * ub_bytes;     // the ring
   const int stages = b.stages;
   const int slot_bytes = b.slot_bytes;
@@ -297,7 +316,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
         }
         __syncwarp();
         if (lane < m)
-          bulk_load(xdst + lane * kXRowBytes,
+          bulk_load(xdst + lane * kXTokBytes,
                     static_cast<const __nv_bfloat16*>(mt.x) + lane * mt.k +
                         static_cast<int64_t>(s) * kSegK,
                     xbytes, full_bar(slot), keep_policy);
@@ -308,6 +327,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
             // per row a box of sb groups from a multiple of sb, as 16-byte copies
             // (k/g % 4 == 0 keeps them aligned), zero past n and past k
             const int sb = decode_scale_box(log2g);
+            const int ss = box_scale_stride(log2g);
             const int64_t gb = g0 - g0 % sb;
             for (int i = 0; i < kRows / 32; ++i) {
               const int r = lane + 32 * i;
@@ -315,18 +335,20 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
               for (int q = 0; q < sb / 4; ++q) {
                 const bool in = row < mt.n && gb + 4 * q < gpr;
                 const float* src = mt.scales + (in ? row * gpr + gb + 4 * q : 0);
-                cp_async16(sdst + (r * sb + 4 * q) * 4, src, in ? 16u : 0u);
+                cp_async16(sdst + (r * ss + 4 * q) * 4, src, in ? 16u : 0u);
               }
             }
           } else {
-            // [256 rows][ng] from group g0, zero past n and past k
+            // [256 rows][ng] from group g0 (rows seg_scale_stride apart), zero past n
+            // and past k
+            const int ss = seg_scale_stride(log2g);
             for (int i = 0; i < kRows / 32; ++i) {
               const int r = lane + 32 * i;
               const int64_t row = row0 + r;
               for (int q = 0; q < ng; ++q) {
                 const bool in = row < mt.n && g0 + q < gpr;
                 const float* src = mt.scales + (in ? row * gpr + g0 + q : 0);
-                cp_async4(sdst + (r * ng + q) * 4, src, in ? 4u : 0u);
+                cp_async4(sdst + (r * ss + q) * 4, src, in ? 4u : 0u);
               }
             }
           }
@@ -392,13 +414,16 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
   const int tok0 = g < m ? g : m - 1;  // tokens past m read token m - 1
   const int tok1 = g + 8 < m ? g + 8 : m - 1;
   const int rl = 32 * wr + g;          // row of tile 0 for C slots 0, 1 (+8: slots 2, 3)
-  // Byte offsets inside a slot that do not change from segment to segment: the
-  // codes of this lane's rows for each of its chunks (the 128-byte swizzle moves
-  // 16-byte chunk j of row r to j ^ (r % 8), and every row of this lane has
-  // r % 8 = g), and its x fragments.
+  // Lane t takes code words t and t + 4 of a chunk's eight (k offsets 16t ..
+  // 16t + 15 and 64 + 16t .. 64 + 16t + 15): the 128-byte swizzle moves 16-byte
+  // chunk j of row r to j ^ (r % 8), so one 32-bit load per word reaches all 32
+  // banks across the warp's eight rows, and the x fragments of the four lanes of
+  // a quarter-warp (bytes 32t .. 32t + 31 of each half chunk) fall on disjoint
+  // banks too.
   constexpr int kMine = kChunks / kSplit;  // chunks of a segment this warp takes
-  auto code_at = [&](int c) { return rl * (kSegK / 4) + (((2 * c + (t >> 1)) ^ g) << 4) + (t & 1) * 8; };
-  auto x_at = [&](int tok, int c) { return tok * kXRowBytes + (128 * c + 32 * t) * 2; };
+  auto code_at = [&](int c) { return rl * (kSegK / 4) + (((2 * c) ^ g) << 4) + 4 * t; };  // word t
+  const int dw4 = (g & 1) ? -16 : 16;  // word t + 4: 16-byte chunk (2c + 1) ^ g = ((2c) ^ g) ^ 1
+  auto x_at = [&](int tok, int c) { return tok * kXTokBytes + 256 * c + 32 * t; };
   // kept in registers up to 8 tokens; recomputed per chunk with two n-tiles,
   // whose accumulators need the registers
   int code_off[kMine], x0_off[kMine];
@@ -426,17 +451,21 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     const int nseg = (k + kSegK - 1) / kSegK;
     // Scale of unit row r and group q: area[r * sstride + q - sq0], the area being
     // the unit buffer (sq0 = 0) or the segment's slot (sq0 = its first stored group).
-    const int sstride = unit_scales ? (k >> log2g)
-                        : mode == kDecodeScale16 ? decode_scale_box(log2g)
-                                                 : (log2g >= 9 ? 1 : kSegK >> log2g);
+    const int sstride = unit_scales ? unit_scale_stride(k >> log2g)
+                        : mode == kDecodeScale16 ? box_scale_stride(log2g)
+                                                 : seg_scale_stride(log2g);
     const float* ubase = nullptr;
     if (unit_scales) {
       const int ub = units_u & 1;
       if (!warp_wait(sfull_bar(ub), (units_u >> 1) & 1, status)) return;
       ubase = reinterpret_cast<const float*>(ubuf + ub * ub_bytes);
     }
-    const int srl = rl * sstride;  // this lane's row of tile 0, C slots 0-1
-    const int s8 = 8 * sstride;    // + 8 rows: C slots 2-3; + 16 rows: the next tile
+    // scale offsets of this lane's rows: tile r, C slots 0-1 (h = 0) and 2-3 (h = 1)
+    int soff[kTiles][2];
+#pragma unroll
+    for (int r = 0; r < kTiles; ++r)
+#pragma unroll
+      for (int h = 0; h < 2; ++h) soff[r][h] = (rl + 16 * r + 8 * h) * sstride;
 #pragma unroll
     for (int r = 0; r < kTiles; ++r)
 #pragma unroll
@@ -444,46 +473,62 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
 
     // Segment s of the unit: its wait (the first one's was the descriptor's), this
     // warp's chunks, the release of the slot. kGuard: the segment reaches past k.
-    // kExact (g >= 128): a chunk lies in one group; its products are accumulated
-    // from zero and folded in with the fp32 scale s (the expanded codes are 2c, so
-    // the sums are twice the output, halved exactly at the store). Otherwise
-    // (g = 32, 64) lane t's offsets 32t .. 32t + 31 of a chunk lie in one group,
+    // kKind 1 (g = 128) and 2 (g >= 256): a chunk lies in one group; its products
+    // are accumulated from zero and folded in with the fp32 scale s (the expanded
+    // codes are 2c, so the sums are twice the output, halved exactly at the store).
+    // kKind 0 (g = 32, 64): the lane's words t and t + 4 each lie in one group,
     // whose bf16(s)/2 multiplies the expanded pairs.
-    auto segment = [&](int s, auto guard, auto exact) -> bool {
+    auto segment = [&](int s, auto guard, auto kind) -> bool {
       constexpr bool kGuard = decltype(guard)::value;
-      constexpr bool kExact = decltype(exact)::value;
+      constexpr int kKind = decltype(kind)::value;
       if (s > 0 && !warp_wait(full_bar(slot), parity, status)) return false;
       const uint8_t* cbase = smem + slot * slot_bytes;
-      const int g0 = (s * kSegK) >> log2g;  // first group of the segment
+      const int kseg = s * kSegK + 128 * kMine * kh;  // first k of this warp's chunks
+      const int g0 = (s * kSegK) >> log2g;             // first group of the segment
       const float* sl = unit_scales ? ubase
                         : reinterpret_cast<const float*>(cbase + kCodeBytes) -
-                              (mode == kDecodeScale16 ? (g0 & -sstride) : g0);
-      const uint8_t* xs = cbase + kCodeBytes + scale_bytes;  // x [m tokens][kSegK]
+                              (mode == kDecodeScale16 ? (g0 & -decode_scale_box(log2g)) : g0);
+      // scales of group q0 + dq(cc) for the lane's four rows
+      const float* sp[kTiles][2];
+      const int q0 = kseg >> log2g;
+#pragma unroll
+      for (int r = 0; r < kTiles; ++r)
+#pragma unroll
+        for (int h = 0; h < 2; ++h) sp[r][h] = sl + soff[r][h] + q0;
+      const uint8_t* xs = cbase + kCodeBytes + scale_bytes;  // x of the m tokens
 #pragma unroll
       for (int cc = 0; cc < kMine; ++cc) {
         const int c = kh * kMine + cc;
-        const int kc = s * kSegK + 128 * c;  // chunk start
+        const int kc = kseg + 128 * cc;  // chunk start
         if (kGuard && kc >= k) break;
-        const bool kin = !kGuard || kc + 32 * t + 32 <= k;  // this lane's 32 offsets lie inside k
+        // k is a multiple of 64: a chunk reaching past k has its first half inside
+        const bool khi = !kGuard || kc + 128 <= k;  // the second half lies inside k
+        // words t (.x) and t + 4 (.y) of rows rl + 16r (h = 0) and + 8 (h = 1)
         uint2 w[kTiles][2];
+        const uint8_t* cw0 = cbase + (kTwoTiles ? code_at(c) : code_off[cc]);
+        const uint8_t* cw1 = cw0 + dw4;
 #pragma unroll
-        for (int r = 0; r < kTiles; ++r) {
-          const uint8_t* cw = cbase + (kTwoTiles ? code_at(c) : code_off[cc]) + r * 16 * (kSegK / 4);
-          w[r][0] = *reinterpret_cast<const uint2*>(cw);
-          w[r][1] = *reinterpret_cast<const uint2*>(cw + 8 * (kSegK / 4));
-        }
-        // past k (a lane of a half chunk) the slot holds no x
+        for (int r = 0; r < kTiles; ++r)
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            w[r][h].x = *reinterpret_cast<const uint32_t*>(cw0 + (16 * r + 8 * h) * (kSegK / 4));
+            w[r][h].y = *reinterpret_cast<const uint32_t*>(cw1 + (16 * r + 8 * h) * (kSegK / 4));
+          }
+        // x of the lane's offsets, xv[0..1] for word t, xv[2..3] for word t + 4
+        // (past k the slot holds no x)
         uint4 xv[4], yv[4];
-        const uint4* xa = reinterpret_cast<const uint4*>(xs + (kTwoTiles ? x_at(tok0, c) : x0_off[cc]));
-        const uint4* xb = reinterpret_cast<const uint4*>(xs + x_at(tok1, c));
+        const uint8_t* xa = xs + (kTwoTiles ? x_at(tok0, c) : x0_off[cc]);
+        const uint8_t* xb = xs + x_at(tok1, c);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-          xv[i] = kin ? xa[i] : make_uint4(0, 0, 0, 0);
-          if (kTwoTiles) yv[i] = kin ? xb[i] : make_uint4(0, 0, 0, 0);
+          const int off = 16 * (i & 1) + 128 * (i >> 1);
+          const bool in = i < 2 || khi;
+          xv[i] = in ? *reinterpret_cast<const uint4*>(xa + off) : make_uint4(0, 0, 0, 0);
+          if (kTwoTiles) yv[i] = in ? *reinterpret_cast<const uint4*>(xb + off) : make_uint4(0, 0, 0, 0);
         }
         const uint32_t* xr = reinterpret_cast<const uint32_t*>(xv);
         const uint32_t* yr = reinterpret_cast<const uint32_t*>(yv);
-        if constexpr (kExact) {
+        if constexpr (kKind != 0) {
           float p[kTiles][4], p1[kTiles][4];
 #pragma unroll
           for (int kb = 0; kb < 8; ++kb) {
@@ -504,12 +549,15 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
               }
             }
           }
+          // group of chunk cc: q0 + cc for g = 128; for g >= 256 the chunks of a
+          // warp's pair share a group (k offsets 256 kh + 128 cc of a 512-aligned
+          // segment), with four chunks one group per two (g = 256) or one in all
+          const int dq = kKind == 1 ? cc : (kMine <= 2 ? 0 : (128 * cc) >> log2g);
           // C slots 0, 1: row rl + 16r, slots 2, 3: row rl + 16r + 8
-          const int q = kc >> log2g;
 #pragma unroll
           for (int r = 0; r < kTiles; ++r) {
-            const float h0 = sl[srl + 2 * r * s8 + q];
-            const float h1 = sl[srl + (2 * r + 1) * s8 + q];
+            const float h0 = sp[r][0][dq];
+            const float h1 = sp[r][1][dq];
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
               acc[r][i] = fmaf(i < 2 ? h0 : h1, p[r][i], acc[r][i]);
@@ -517,16 +565,20 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
             }
           }
         } else {
-          const int q = (kc + 32 * t) >> log2g;
+          // the lane's words t and t + 4 lie in groups qa and qb
+          const int qa = (kc + 16 * t) >> log2g, qb = (kc + 64 + 16 * t) >> log2g;
 #pragma unroll
           for (int r = 0; r < kTiles; ++r) {
-            const uint32_t hs0 = kin ? half_scale_bf16x2(sl[srl + 2 * r * s8 + q]) : 0u;
-            const uint32_t hs1 = kin ? half_scale_bf16x2(sl[srl + (2 * r + 1) * s8 + q]) : 0u;
+            const uint32_t hs0a = half_scale_bf16x2(sl[soff[r][0] + qa]);
+            const uint32_t hs1a = half_scale_bf16x2(sl[soff[r][1] + qa]);
+            const uint32_t hs0b = khi ? half_scale_bf16x2(sl[soff[r][0] + qb]) : 0u;
+            const uint32_t hs1b = khi ? half_scale_bf16x2(sl[soff[r][1] + qb]) : 0u;
 #pragma unroll
             for (int kb = 0; kb < 8; ++kb) {
               const int j = 2 * (kb & 3);
               const uint32_t u0 = kb < 4 ? w[r][0].x : w[r][0].y;
               const uint32_t u1 = kb < 4 ? w[r][1].x : w[r][1].y;
+              const uint32_t hs0 = kb < 4 ? hs0a : hs0b, hs1 = kb < 4 ? hs1a : hs1b;
               const uint32_t a0 = bmul2(pair_bits(u0, j, mul[j]), hs0);
               const uint32_t a1 = bmul2(pair_bits(u1, j, mul[j]), hs1);
               const uint32_t a2 = bmul2(pair_bits(u0, j + 1, mul[j + 1]), hs0);
@@ -546,20 +598,22 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
       return true;
     };
     bool ok = true;
-    auto run = [&](auto exact) {
+    auto run = [&](auto kind) {
       if constexpr (kTwoTiles) {
         // (two n-tiles: no register room for a second chunk body)
-        for (int s = 0; s < nseg && ok; ++s) ok = segment(s, std::true_type{}, exact);
+        for (int s = 0; s < nseg && ok; ++s) ok = segment(s, std::true_type{}, kind);
       } else {
-        for (int s = 0; s < nfull && ok; ++s) ok = segment(s, std::false_type{}, exact);
-        if (ok && nfull < nseg) ok = segment(nfull, std::true_type{}, exact);
+        for (int s = 0; s < nfull && ok; ++s) ok = segment(s, std::false_type{}, kind);
+        if (ok && nfull < nseg) ok = segment(nfull, std::true_type{}, kind);
       }
     };
     const bool exact = log2g >= 7;
-    if (exact)
-      run(std::true_type{});
+    if (log2g == 7)
+      run(std::integral_constant<int, 1>{});
+    else if (exact)
+      run(std::integral_constant<int, 2>{});
     else
-      run(std::false_type{});
+      run(std::integral_constant<int, 0>{});
     if (!ok) return;
     if (unit_scales) {
       if (lane == 0) mbar_arrive(sempty_bar(units_u & 1));
@@ -676,19 +730,21 @@ cudaError_t launch_decode(DecodeBatch& b, int num_sms, cudaStream_t stream) {
     const int lg = b.mats[d].log2g;
     const int64_t gpr = b.mats[d].k >> lg;
     if (b.mats[d].scale_mode == kDecodeScaleUnit) {
-      ugroups = gpr > ugroups ? gpr : ugroups;
+      const int64_t w = unit_scale_stride(static_cast<int>(gpr));  // gpr <= 32 in this mode
+      ugroups = w > ugroups ? w : ugroups;
     } else {
-      const int w = b.mats[d].scale_mode == kDecodeScale16 ? decode_scale_box(lg) : (lg >= 9 ? 1 : kSegK >> lg);
+      const int w = b.mats[d].scale_mode == kDecodeScale16 ? box_scale_stride(lg) : seg_scale_stride(lg);
       sgroups = w > sgroups ? w : sgroups;
     }
   }
   b.ubuf_bytes = static_cast<int32_t>(kRows * ugroups * 4);
   b.scale_bytes = kRows * sgroups * 4;
-  b.slot_bytes = (kCodeBytes + b.scale_bytes + b.m * kXRowBytes + 1023) & ~1023;
-  const int fit = (kSmemLimit - 1024 - kHeadBytes - kRedBytes - 2 * b.ubuf_bytes) / b.slot_bytes;
+  b.slot_bytes = (kCodeBytes + b.scale_bytes + b.m * kXTokBytes + 1023) & ~1023;
+  const int red = b.m > 8 ? red_bytes<true>() : red_bytes<false>();
+  const int fit = (kSmemLimit - 1024 - kHeadBytes - red - 2 * b.ubuf_bytes) / b.slot_bytes;
   b.stages = fit < kMaxStages ? fit : kMaxStages;
   if (b.stages < 2) return cudaErrorInvalidValue;
-  const int smem = 1024 + kHeadBytes + kRedBytes + 2 * b.ubuf_bytes + b.stages * b.slot_bytes;
+  const int smem = 1024 + kHeadBytes + red + 2 * b.ubuf_bytes + b.stages * b.slot_bytes;
   uint32_t* sched = dsched_base();
   if (sched == nullptr) return cudaErrorInvalidSymbol;
   sched += 2 * (seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
