@@ -116,7 +116,10 @@ TQ_API tq_status tq_quantize_batched(const tq_quant_desc* descs, int32_t count, 
  *   y            out: [m][n], fp32 (TQ_OUT_F32) or bf16 (TQ_OUT_BF16).
  *   Requires k % 64 == 0 and k % g == 0; n >= 1 when m >= 1.
  *   m <= 16 runs the decode kernel, larger m the tensor-core GEMM; both expand
- *   the codes on chip to bf16 (bf16(s) * code) and accumulate in fp32.
+ *   the codes on chip and accumulate in fp32 (the decode kernel folds the fp32
+ *   scale into each group's sum for g >= 128, the others multiply the expanded
+ *   codes by bf16(s)). The decode kernel takes k <= 2^30 and n < 2^31
+ *   (TQ_ERR_UNSUPPORTED beyond).
  */
 TQ_API tq_status tq_linear_fwd(const void* x, int64_t m, int64_t k,
                         const uint32_t* codes, const float* scales, int64_t n, int32_t g,

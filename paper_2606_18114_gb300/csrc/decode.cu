@@ -440,7 +440,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     // The first segment of a unit carries the unit's descriptor: everything that
     // depends on the matrix is decided here once, so that per segment a warp runs
     // one wait, its chunks and one arrival.
-    if (!warp_wait(full_bar(slot), parity, status)) return;
+    if (!lanes_wait(full_bar(slot), parity, status)) return;
     const SegInfo si = info[slot];
     if (si.mat < 0) break;
     const int k = si.k;
@@ -457,7 +457,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     const float* ubase = nullptr;
     if (unit_scales) {
       const int ub = units_u & 1;
-      if (!warp_wait(sfull_bar(ub), (units_u >> 1) & 1, status)) return;
+      if (!lanes_wait(sfull_bar(ub), (units_u >> 1) & 1, status)) return;
       ubase = reinterpret_cast<const float*>(ubuf + ub * ub_bytes);
     }
     // scale offsets of this lane's rows: tile r, C slots 0-1 (h = 0) and 2-3 (h = 1)
@@ -481,7 +481,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     auto segment = [&](int s, auto guard, auto kind) -> bool {
       constexpr bool kGuard = decltype(guard)::value;
       constexpr int kKind = decltype(kind)::value;
-      if (s > 0 && !warp_wait(full_bar(slot), parity, status)) return false;
+      if (s > 0 && !lanes_wait(full_bar(slot), parity, status)) return false;
       const uint8_t* cbase = smem + slot * slot_bytes;
       const int kseg = s * kSegK + 128 * kMine * kh;  // first k of this warp's chunks
       const int g0 = (s * kSegK) >> log2g;             // first group of the segment
@@ -626,7 +626,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
       const uint32_t ph = (units_r >> 1) & 1;
       float* rb = red + ((pb * kRowWarps + wr) * 32 + lane) * (kTiles * 4);
       if (kh == 1) {
-        if (units_r >= 2 && !warp_wait(rempty_bar(wr, pb), ph ^ 1u, status)) return;
+        if (units_r >= 2 && !lanes_wait(rempty_bar(wr, pb), ph ^ 1u, status)) return;
 #pragma unroll
         for (int r = 0; r < kTiles; ++r)
 #pragma unroll
@@ -634,7 +634,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(rfull_bar(wr, pb));
       } else {
-        if (!warp_wait(rfull_bar(wr, pb), ph, status)) return;
+        if (!lanes_wait(rfull_bar(wr, pb), ph, status)) return;
 #pragma unroll
         for (int r = 0; r < kTiles; ++r)
 #pragma unroll
@@ -646,31 +646,37 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     }
     if (kh == 0) {
       // C fragment of tile r: rows rl + 16r (slots 0, 1) and + 8 (2, 3), tokens 2t, 2t + 1
-      const int64_t n = si.n;
-      const bool ybf16 = (si.mode >> 8) != 0;
+      const int n = si.n;  // rows (< 2^31) and row0 + 256 <= n + 255 fit in 32 bits
       const float post = exact ? 0.5f : 1.f;
-      auto store = [&](int token, int64_t row, float v) {
-        if (token < m && row < n) {
-          if (ybf16)
-            static_cast<__nv_bfloat16*>(si.y)[token * n + row] = __float2bfloat16_rn(post * v);
-          else
-            static_cast<float*>(si.y)[token * n + row] = post * v;
+      auto put = [&](auto* y) {
+        using T = std::remove_pointer_t<decltype(y)>;
+        auto store = [&](int token, int row, float v) {
+          if (token < m && row < n) {
+            if constexpr (std::is_same_v<T, float>)
+              y[static_cast<int64_t>(token) * n + row] = post * v;
+            else
+              y[static_cast<int64_t>(token) * n + row] = __float2bfloat16_rn(post * v);
+          }
+        };
+#pragma unroll
+        for (int r = 0; r < kTiles; ++r) {
+          const int ra = si.row0 + rl + 16 * r, rb = ra + 8;
+          store(2 * t, ra, acc[r][0]);
+          store(2 * t + 1, ra, acc[r][1]);
+          store(2 * t, rb, acc[r][2]);
+          store(2 * t + 1, rb, acc[r][3]);
+          if (kTwoTiles) {
+            store(8 + 2 * t, ra, acc1[r][0]);
+            store(8 + 2 * t + 1, ra, acc1[r][1]);
+            store(8 + 2 * t, rb, acc1[r][2]);
+            store(8 + 2 * t + 1, rb, acc1[r][3]);
+          }
         }
       };
-#pragma unroll
-      for (int r = 0; r < kTiles; ++r) {
-        const int64_t ra = si.row0 + rl + 16 * r, rb = ra + 8;
-        store(2 * t, ra, acc[r][0]);
-        store(2 * t + 1, ra, acc[r][1]);
-        store(2 * t, rb, acc[r][2]);
-        store(2 * t + 1, rb, acc[r][3]);
-        if (kTwoTiles) {
-          store(8 + 2 * t, ra, acc1[r][0]);
-          store(8 + 2 * t + 1, ra, acc1[r][1]);
-          store(8 + 2 * t, rb, acc1[r][2]);
-          store(8 + 2 * t + 1, rb, acc1[r][3]);
-        }
-      }
+      if ((si.mode >> 8) != 0)
+        put(static_cast<__nv_bfloat16*>(si.y));
+      else
+        put(static_cast<float*>(si.y));
     }
   }
 }

@@ -106,6 +106,16 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, int* st
   return ok != 0;
 }
 
+// Wait by every lane of a converged warp: in the common case (the phase has
+// completed) one test for the whole warp, with no broadcast; each lane's own
+// wait orders its later reads. The lanes poll in lockstep on the same word, so
+// they agree; the vote makes the outcome uniform in any case.
+__device__ __forceinline__ bool lanes_wait(uint32_t bar, uint32_t parity, int* status) {
+  if (mbar_test_wait(bar, parity)) return true;
+  const bool ok = mbar_wait(bar, parity, status);
+  return __all_sync(0xffffffffu, ok);
+}
+
 __device__ __forceinline__ bool warp_wait2(uint32_t bar0, uint32_t parity0, uint32_t bar1,
                                            uint32_t parity1, int* status) {
   int ok = 1;

@@ -265,6 +265,7 @@ tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
       continue;
     }
     if (d.n >= (int64_t(1) << 31)) return fail(TQ_ERR_UNSUPPORTED, "too many decode rows");
+    if (d.k > (int64_t(1) << 30)) return fail(TQ_ERR_UNSUPPORTED, "decode reduction longer than 2^30");
     const int log2g = log2_group(d.g);
     const int64_t gpr = d.k >> log2g;
     TQ_TRY(decode_map(0, d.codes, d.n, d.k, 0, &b.maps[used]));
