@@ -200,7 +200,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   int slot = 0;
   uint32_t parity = 0;
   for (;;) {
-    if (!warp_wait(full_bar(slot), parity, status)) return;
+    if (!lanes_wait(full_bar(slot), parity, status)) return;
     const int64_t ls = stage_of[slot];
     if (ls < 0) return;
     const QuantMat& mt = b.mats[kMax == 1 ? 0 : mat_of[slot]];

@@ -234,7 +234,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < my_tiles; ++i) {
       const int acc = i % kAcc;
       const uint32_t aph = (i / kAcc) & 1;
-      if (!warp_wait(accfull_bar(acc), aph, status)) break;
+      if (!lanes_wait(accfull_bar(acc), aph, status)) break;
       tc_fence_after();
       const int64_t row = tile_r0(i) + quad * 32 + lane;
       const int64_t m0 = tile_m0(i);
@@ -300,9 +300,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (L::kReleaseViaSmem) {
         if (it < kAS) return true;
         const int j = it - kAS;
-        return warp_wait(empty_bar(j % kSmem), (j / kSmem) & 1, status);
+        return lanes_wait(empty_bar(j % kSmem), (j / kSmem) & 1, status);
       }
-      return warp_wait(aempty_bar(it % kAS), ((it / kAS) & 1) ^ 1, status);
+      return lanes_wait(aempty_bar(it % kAS), ((it / kAS) & 1) ^ 1, status);
     };
     auto publish = [&](int as, const uint32_t* a) {
       tc_fence_after();
@@ -335,7 +335,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         p1 = load_sc(pre);
         // Expand as soon as the codes have landed; only the tensor-memory store
         // waits for the A stage.
-        if (!warp_wait(full_bar(s), (it / kSmem) & 1, status)) break;
+        if (!lanes_wait(full_bar(s), (it / kSmem) & 1, status)) break;
         const uint4 cw = *reinterpret_cast<const uint4*>(smem + s * L::kStageBytes + L::kBBytes +
                                                          r_local * 32 + wg * 16);
         const uint32_t hs_lo = half_scale_pair(sc.x, sc.x);
@@ -380,7 +380,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           sb[lane] = __float2bfloat16_rn(0.5f * sc.x);
           sb[lane + 32] = __float2bfloat16_rn(0.5f * sc.y);
           __syncwarp();
-          if (!warp_wait(full_bar(s), (it / kSmem) & 1, status)) break;
+          if (!lanes_wait(full_bar(s), (it / kSmem) & 1, status)) break;
           const uint4 cw = *reinterpret_cast<const uint4*>(smem + s * L::kStageBytes + L::kBBytes +
                                                            r_local * 32 + wg * 16);
           const uint4* sp = reinterpret_cast<const uint4*>(sb);  // 32 pairs of rows n
@@ -414,7 +414,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         sb[lane] = __float2bfloat16_rn(0.5f * sc.x);
         sb[lane + 32] = __float2bfloat16_rn(0.5f * sc.y);
         __syncwarp();
-        if (!warp_wait(full_bar(s), (it / kSmem) & 1, status)) break;
+        if (!lanes_wait(full_bar(s), (it / kSmem) & 1, status)) break;
         const uint32_t* tile =
             reinterpret_cast<const uint32_t*>(smem + s * L::kStageBytes + L::kBBytes) + wg * 64 * 8;
         const uint32_t* spair = reinterpret_cast<const uint32_t*>(sb);
