@@ -138,6 +138,7 @@ struct DwArgs {
 
 constexpr int kDwTileK = 128;  // lanes: input features
 constexpr int kDwTileN = 256;  // columns: output features
+constexpr int kDwMaxCtas = 160;  // grid cap (stream-K workspace: two tiles per CTA)
 size_t dw_smem_bytes();
 
 // tmap_x: bf16 x [m][k] box {64, 64}; tmap_dy: bf16 dy [m][n] box {64, 64};

@@ -106,6 +106,12 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, int* st
   return ok != 0;
 }
 
+// Hardware barrier `id` (1..15) among `count` threads of the CTA (a multiple of
+// 32; the warps that take part all reach it).
+__device__ __forceinline__ void named_bar_sync(uint32_t id, uint32_t count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 // Wait by every lane of a converged warp: in the common case (the phase has
 // completed) one test for the whole warp, with no broadcast; each lane's own
 // wait orders its later reads. The lanes poll in lockstep on the same word, so

@@ -240,6 +240,28 @@ def test_dw_accumulate_and_single_outputs(tq):
     check_close(dx2, O.linear_bwd_dx(dy, w_hat), "dX only")
 
 
+@pytest.mark.parametrize("m", [64, 640, 1000])
+@pytest.mark.parametrize("accumulate", [False, True])
+def test_dw_stream_k_tail(tq, m, accumulate):
+    """dW over more 128 x 256 tiles than SMs (10 x 17 = 170): the tiles past the last
+    whole wave are cut into runs of k-blocks, one per CTA, and summed in k order by
+    the CTA that completes each tile. m = 64 leaves fewer tail k-blocks than CTAs
+    (every tile whole), m = 640 cuts tiles into many pieces, m = 1000 ends on a
+    ragged k-block. Full comparison with the oracle."""
+    n, k, g = 4160, 1280, 128
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=11, dy_std=1e-2)
+    xd, dyd = x.cuda(), dy.cuda()
+    base = torch.randn(n, k, device="cuda", dtype=torch.float32) if accumulate else None
+    dw = base.clone() if accumulate else None
+    for _ in range(2):  # the second launch reuses the reset tail counters
+        out = base.clone() if accumulate else dw
+        _, dw = tq.linear_bwd(dyd, xd, codes, s, k, g, want_dx=False, dw=out,
+                              accumulate_dw=accumulate)
+        tq.device_status()
+        got = to_np(dw).astype(np.float64) - (to_np(base).astype(np.float64) if accumulate else 0)
+        check_close(got, O.linear_bwd_dw(dy, x), f"dW m={m} accumulate={accumulate}")
+
+
 def test_empty_sizes(tq):
     codes = torch.zeros((64, 256 // 16), dtype=torch.int32, device="cuda")
     s = torch.zeros((64, 2), dtype=torch.float32, device="cuda")
