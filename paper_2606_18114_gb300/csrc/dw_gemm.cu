@@ -26,7 +26,8 @@
 // each piece's fp32 sum written to the workspace (two slots per CTA: the piece
 // that opens its run and the one that closes it); the CTA that completes the last
 // piece (a per-tile counter) adds the pieces in k order and writes dW. No CTA
-// waits for another.
+// waits for another. The tail's CTAs read their runs' tokens at different
+// offsets, so there dy is kept in L2 (evict-last) like x.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -190,7 +191,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int c = 0; c < 4; ++c)
             tma_load_2d_hint(b + c * kBox, &tmap_dy, full_bar(s), static_cast<int32_t>(n0 + 64 * c),
-                             mrow, stream);
+                             mrow, wi.sk < 0 ? stream : keep);
           ++issued;
         }
       }
