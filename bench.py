@@ -373,6 +373,119 @@ def quantize_sweep(tq, steps, warmup):
     return {"ms": round(ms, 3), "GB/s": round(nbytes / ms / 1e6, 1), "bytes": nbytes}
 
 
+def out_proj_step(tq, steps, warmup):
+    """The same step on the out_proj shape (W [2048, 4096], X [16384, 4096])."""
+    p = Prefill(tq, OUT_PROJ[0], OUT_PROJ[1], M_PREFILL, G, seed=8)
+    total_ms, per = time_prefill(p, steps, warmup, 1)
+    ms = total_ms / steps
+    gemm = 2.0 * p.m * p.n * p.k
+    out = {"ms": round(ms, 4), "TFLOP/s": round(p.flops / ms / 1e9, 1)}
+    for name in ("fwd", "dx", "dw"):
+        out[name] = {"ms": round(per[name], 4), "TFLOP/s": round(gemm / per[name] / 1e9, 1)}
+    out["quantize"] = {"ms": round(per["quantize"], 4),
+                       "GB/s": round(p.quantize_bytes() / per["quantize"] / 1e6, 1)}
+    del p
+    return out
+
+
+def student_t3(shape, gen, std):
+    """Student-t with 3 degrees of freedom scaled to standard deviation std: z / sqrt(chi2_3 / 3),
+    the variance of t_3 being 3."""
+    z = torch.randn(shape, generator=gen, device="cuda")
+    c = sum(torch.randn(shape, generator=gen, device="cuda") ** 2 for _ in range(3)) / 3.0
+    return z / c.sqrt() * (std / math.sqrt(3.0))
+
+
+def g_sweep(tq):
+    """The 48-block sweep at batch 8 x seq 2048 for every group size and both weight
+    distributions: per (distribution, g) one batched requantize of the 96 projections,
+    then per projection the codes transpose, forward, dX and dW. X and dY are shared by
+    the layers of a projection type (the GEMMs are compute-bound)."""
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(5)
+    shapes = [IN_PROJ, OUT_PROJ] * N_LAYERS
+    act = {}
+    for n, k in (IN_PROJ, OUT_PROJ):
+        act[(n, k)] = dict(
+            x=torch.randn((M_PREFILL, k), generator=gen, device="cuda").to(torch.bfloat16),
+            dy=(torch.randn((M_PREFILL, n), generator=gen, device="cuda") * 1e-2).to(torch.bfloat16),
+            y=torch.empty((M_PREFILL, n), device="cuda"),
+            dx=torch.empty((M_PREFILL, k), device="cuda"),
+            dw=torch.empty((n, k), device="cuda"))
+    flops = sum(3 * 2.0 * M_PREFILL * n * k for n, k in shapes)
+    pk, _ = peaks()
+    res = {}
+    for dist in ("gauss", "t3"):
+        ws = [(torch.randn(sh, generator=gen, device="cuda") * 0.02) if dist == "gauss"
+              else student_t3(sh, gen, 0.02) for sh in shapes]
+        codes = [torch.empty((n, k // 16), dtype=torch.int32, device="cuda") for n, k in shapes]
+        codes_t = [torch.empty((k, 4 * ((n + 63) // 64)), dtype=torch.int32, device="cuda")
+                   for n, k in shapes]
+        for g in (32, 64, 128, 256, 512):
+            sc = [torch.empty((n, k // g), device="cuda") for n, k in shapes]
+            zs = [torch.empty((n, k // g), dtype=torch.int32, device="cuda") for n, k in shapes]
+            arr = tq.quant_batch([(w, c, s_, z) for w, c, s_, z in zip(ws, codes, sc, zs)])
+
+            def gemms():
+                for (n, k), c, ct, s_ in zip(shapes, codes, codes_t, sc):
+                    a = act[(n, k)]
+                    tq.codes_transpose(c, k, out=ct)
+                    tq.linear_fwd(a["x"], c, s_, g, y=a["y"])
+                    tq.linear_bwd(a["dy"], a["x"], c, s_, k, g, want_dw=False, dx=a["dx"], codes_t=ct)
+                    tq.linear_bwd(a["dy"], a["x"], c, s_, k, g, want_dx=False, dw=a["dw"])
+
+            tq.quantize_batched(arr, g)
+            gemms()
+            torch.cuda.synchronize()
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            ev[0].record()
+            tq.quantize_batched(arr, g)
+            ev[1].record()
+            gemms()
+            ev[2].record()
+            torch.cuda.synchronize()
+            tq.device_status()
+            q_ms, g_ms = ev[0].elapsed_time(ev[1]), ev[1].elapsed_time(ev[2])
+            numel = sum(n * k for n, k in shapes)
+            qbytes = numel * 4 + numel // 4 + 2 * 4 * numel // g
+            zero = sum(int(z.sum(dtype=torch.int64)) for z in zs) / numel
+            ach = flops / g_ms / 1e9
+            res[f"{dist}_g{g}"] = {
+                "quantize_ms": round(q_ms, 3), "quantize_GB/s": round(qbytes / q_ms / 1e6, 1),
+                "quantize_frac": round(qbytes / q_ms / 1e6 / pk["hbm_gbs"], 4),
+                "gemms_ms": round(g_ms, 2), "TFLOP/s": round(ach, 1),
+                "frac": round(ach / pk["bf16_tflops"], 4), "zero_ratio": round(zero, 4)}
+            del sc, zs, arr
+        del ws, codes, codes_t
+    res["note"] = ("per (distribution, g): one batched requantize of the 96 projections, then "
+                   "codes transpose + forward + dX + dW of every projection; "
+                   f"{flops / 1e12:.2f} TFLOP of GEMMs per sweep")
+    return res
+
+
+def cublas_context(tq):
+    """cuBLAS bf16 dense GEMM of the forward's shape (Y = X W^T, 16384 x 8512 x 2048):
+    context for the tensor-core fraction, not part of the path."""
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(3)
+    x = torch.randn((M_PREFILL, IN_PROJ[1]), generator=gen, device="cuda").to(torch.bfloat16)
+    w = torch.randn(IN_PROJ, generator=gen, device="cuda").to(torch.bfloat16)
+    for _ in range(3):
+        torch.matmul(x, w.t())
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(20):
+        torch.matmul(x, w.t())
+    t1.record()
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1) / 20
+    return {"ms": round(ms, 4),
+            "TFLOP/s": round(2.0 * M_PREFILL * IN_PROJ[0] * IN_PROJ[1] / ms / 1e9, 1),
+            "note": "torch.matmul bf16 (cuBLAS), bf16 output; context only"}
+
+
 # ------------------------------------------------------------------ oracle (CPU)
 def blas_threads():
     try:
@@ -573,6 +686,9 @@ def main():
         line["extra"] = {
             "decode_48_layers": decode_sweep(tq, (1, 4, 16), 20, 3),
             "quantize_48_layers_g128": quantize_sweep(tq, 5, 2),
+            "out_proj_step": out_proj_step(tq, 200, 10),
+            "sweep_48_layers": g_sweep(tq),
+            "cublas_bf16_fwd_shape": cublas_context(tq),
             "hbm_peak_gbs": pk["hbm_gbs"],
         }
     if rank == 0 and world == 1 and not args.no_cpu:
