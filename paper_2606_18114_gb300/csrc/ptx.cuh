@@ -336,6 +336,12 @@ __device__ __forceinline__ void tmem_ld_wait(uint32_t (&r)[32]) {
                : "memory");
 }
 
+// After a tcgen05.wait::ld issued elsewhere: ties 16 more registers of earlier
+// loads to that point (an empty volatile statement, ordered after the wait).
+__device__ __forceinline__ void tmem_regs_ready16(uint32_t (&r)[16]) {
+  asm volatile("" : TQ_RW8(0), TQ_RW8(8));
+}
+
 #undef TQ_R8
 #undef TQ_W8
 #undef TQ_RW8

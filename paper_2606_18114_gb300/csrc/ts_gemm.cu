@@ -242,22 +242,31 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t d = tmem_base + acc * BN + lane_off;
       // element (m0 + c + t, row) of out; tokens beyond m are not stored
       const int mvalid = static_cast<int>(m - m0 < BN ? m - m0 : BN);
+      // four 16-column loads in flight per wait
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 16) {
-        uint32_t v[16];
-        tmem_ld16(d + c, v);
-        tmem_ld_wait16(v);
+      for (int c0 = 0; c0 < BN; c0 += 64) {
+        uint32_t v[4][16];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) tmem_ld16(d + c0 + 16 * q, v[q]);
+        tmem_ld_wait16(v[0]);
+        tmem_regs_ready16(v[1]);
+        tmem_regs_ready16(v[2]);
+        tmem_regs_ready16(v[3]);
         if (row < rows) {
-          if (args.out_bf16) {
-            __nv_bfloat16* p = static_cast<__nv_bfloat16*>(args.out) + (m0 + c) * rows + row;
 #pragma unroll
-            for (int t = 0; t < 16; ++t, p += rows)
-              if (c + t < mvalid) *p = __float2bfloat16_rn(__uint_as_float(v[t]));
-          } else {
-            float* p = static_cast<float*>(args.out) + (m0 + c) * rows + row;
+          for (int q = 0; q < 4; ++q) {
+            const int c = c0 + 16 * q;
+            if (args.out_bf16) {
+              __nv_bfloat16* p = static_cast<__nv_bfloat16*>(args.out) + (m0 + c) * rows + row;
 #pragma unroll
-            for (int t = 0; t < 16; ++t, p += rows)
-              if (c + t < mvalid) *p = __uint_as_float(v[t]);
+              for (int t = 0; t < 16; ++t, p += rows)
+                if (c + t < mvalid) *p = __float2bfloat16_rn(__uint_as_float(v[q][t]));
+            } else {
+              float* p = static_cast<float*>(args.out) + (m0 + c) * rows + row;
+#pragma unroll
+              for (int t = 0; t < 16; ++t, p += rows)
+                if (c + t < mvalid) *p = __uint_as_float(v[q][t]);
+            }
           }
         }
       }
