@@ -357,25 +357,28 @@ def test_linear_mamba2_prefill_sampled(tq, proj):
 _SWEEP = {}
 
 
-def _sweep_inputs(dist):
-    """in_proj-shaped W (per distribution) and one X / dY shared by the sweep."""
-    n, k = synth.MAMBA2_1P3B["in_proj"]
-    if "xdy" not in _SWEEP:
+def _sweep_inputs(proj, dist):
+    """W of the projection's shape (per distribution) and one X / dY per projection,
+    shared by the sweep's group sizes."""
+    n, k = synth.MAMBA2_1P3B[proj]
+    if (proj, "xdy") not in _SWEEP:
+        _SWEEP.clear()  # one projection's inputs at a time (the host arrays are large)
         x = synth.activations_bf16(16384, k, seed=5, stream="x")
         dy = synth.activations_bf16(16384, n, seed=5, std=1e-2, stream="dy")
-        _SWEEP["xdy"] = (x, dy, x.cuda(), dy.cuda())
-    if dist not in _SWEEP:
-        _SWEEP[dist] = synth.latent_weights(n, k, seed=5, dist=dist)
-    return (_SWEEP[dist],) + _SWEEP["xdy"]
+        _SWEEP[(proj, "xdy")] = (x, dy, x.cuda(), dy.cuda())
+    if (proj, dist) not in _SWEEP:
+        _SWEEP[(proj, dist)] = synth.latent_weights(n, k, seed=5, dist=dist)
+    return (_SWEEP[(proj, dist)],) + _SWEEP[(proj, "xdy")]
 
 
 @pytest.mark.parametrize("dist", ["gauss", "t3"])
 @pytest.mark.parametrize("g", [32, 64, 128, 256, 512])
-def test_prefill_sweep_all_group_sizes(tq, g, dist):
-    """One full in_proj step (quantize, Y, dX on the transposed codes, dW) at
-    M = 16384 for each group size and weight distribution; outputs checked on
-    sampled rows, every group's code and scale checked in full."""
-    w, x, dy, xd, dyd = _sweep_inputs(dist)
+@pytest.mark.parametrize("proj", ["in_proj", "out_proj"])
+def test_prefill_sweep_all_group_sizes(tq, proj, g, dist):
+    """One full projection step (quantize, Y, dX on the transposed codes, dW) at
+    M = 16384 for each projection, group size and weight distribution; outputs
+    checked on sampled rows, every group's code and scale checked in full."""
+    w, x, dy, xd, dyd = _sweep_inputs(proj, dist)
     n, k = w.shape
     ref = O.quantize(w, g)
     codes, s, z = _quant(tq, w, g)
@@ -390,7 +393,7 @@ def test_prefill_sweep_all_group_sizes(tq, g, dist):
     rows = np.sort(rs.choice(16384, 32, replace=False))
     nrows = np.sort(rs.choice(n, 32, replace=False))
     sel = torch.from_numpy(rows).cuda()
-    check_close(to_np(y[sel]), O.linear_fwd(x, w_hat, rows), f"Y rows g={g} {dist}")
-    check_close(to_np(dx[sel]), O.linear_bwd_dx(dy, w_hat, rows), f"dX rows g={g} {dist}")
+    check_close(to_np(y[sel]), O.linear_fwd(x, w_hat, rows), f"Y rows {proj} g={g} {dist}")
+    check_close(to_np(dx[sel]), O.linear_bwd_dx(dy, w_hat, rows), f"dX rows {proj} g={g} {dist}")
     check_close(to_np(dw[torch.from_numpy(nrows).cuda()]), O.linear_bwd_dw(dy, x, nrows),
-                f"dW rows g={g} {dist}")
+                f"dW rows {proj} g={g} {dist}")
