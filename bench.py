@@ -463,6 +463,57 @@ def g_sweep(tq):
     return res
 
 
+def adamw_sweep(tq, steps, warmup):
+    """tq_adamw_requantize (AdamW step + requantize, g = 128) on the in_proj matrix
+    alone and over the 96 projections of the 48 blocks (one launch each): per weight
+    16 B read (w, grad, m, v) and 12 B + codes + scale and count written."""
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(31)
+    pk, _ = peaks()
+    hp = dict(lr=2.5e-4, beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.01)
+
+    def state(n, k):
+        w = torch.randn((n, k), generator=gen, device="cuda") * 0.02
+        g = torch.randn((n, k), generator=gen, device="cuda") * 1e-3
+        m = torch.zeros((n, k), device="cuda")
+        v = torch.zeros((n, k), device="cuda")
+        out = (torch.empty((n, k // 16), dtype=torch.int32, device="cuda"),
+               torch.empty((n, k // G), device="cuda"),
+               torch.empty((n, k // G), dtype=torch.int32, device="cuda"))
+        return w, g, m, v, out
+
+    def per_weight_bytes():
+        return 28 + 0.25 + 8.0 / G
+
+    res = {}
+    for label, shapes in (("in_proj", [IN_PROJ]), ("48_layers", [IN_PROJ, OUT_PROJ] * N_LAYERS)):
+        mats = [state(n, k) for n, k in shapes]
+        t = [0]
+
+        def run():
+            t[0] += 1
+            for w, g, m, v, out in mats:
+                tq.adamw_requantize(w, g, m, v, G, step=t[0], out=out, **hp)
+
+        for _ in range(warmup):
+            run()
+        torch.cuda.synchronize()
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record()
+        for _ in range(steps):
+            run()
+        t1.record()
+        torch.cuda.synchronize()
+        ms = t0.elapsed_time(t1) / steps
+        nbytes = sum(n * k for n, k in shapes) * per_weight_bytes()
+        res[label] = {"ms": round(ms, 4), "GB/s": round(nbytes / ms / 1e6, 1),
+                      "frac": round(nbytes / ms / 1e6 / pk["hbm_gbs"], 4), "bytes": int(nbytes)}
+        del mats
+    tq.device_status()
+    return res
+
+
 def cublas_context(tq):
     """cuBLAS bf16 dense GEMM of the forward's shape (Y = X W^T, 16384 x 8512 x 2048):
     context for the tensor-core fraction, not part of the path."""
@@ -574,17 +625,31 @@ def run_only(args):
         res = decode_sweep(tq, (1,), args.steps, args.warmup)
         print(json.dumps({"only": "decode", **res}), flush=True)
         return
+    if args.only == "adamw":
+        n, k = IN_PROJ
+        w = torch.randn((n, k), device="cuda") * 0.02
+        gr = torch.randn((n, k), device="cuda") * 1e-3
+        m = torch.zeros((n, k), device="cuda")
+        v = torch.zeros((n, k), device="cuda")
+        step = [0]
+
+        def upd():
+            step[0] += 1
+            tq.adamw_requantize(w, gr, m, v, G, lr=2.5e-4, step=step[0])
+        calls = {"adamw": upd}
+    else:
+        calls = {}
     p = Prefill(tq, IN_PROJ[0], IN_PROJ[1], M_PREFILL, G, seed=7)
     tq.quantize(p.w, p.g, out=(p.codes, p.s, p.z))
     tq.codes_transpose(p.codes, p.k, out=p.codes_t)
-    calls = {
+    calls.update({
         "quantize": lambda: tq.quantize(p.w, p.g, out=(p.codes, p.s, p.z)),
         "transpose": lambda: tq.codes_transpose(p.codes, p.k, out=p.codes_t),
         "fwd": lambda: tq.linear_fwd(p.x, p.codes, p.s, p.g, y=p.y),
         "dx": lambda: tq.linear_bwd(p.dy, p.x, p.codes, p.s, p.k, p.g, want_dw=False, dx=p.dx,
                                     codes_t=p.codes_t),
         "dw": lambda: tq.linear_bwd(p.dy, p.x, p.codes, p.s, p.k, p.g, want_dx=False, dw=p.dw),
-    }
+    })
     fn = calls[args.only]
     for _ in range(args.warmup):
         fn()
@@ -610,7 +675,7 @@ def main():
     ap.add_argument("--impl", default="tq", choices=["tq", "reference"])
     ap.add_argument("--no-extra", action="store_true", help="skip decode/quantize sweeps")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
-    ap.add_argument("--only", choices=["quantize", "transpose", "fwd", "dx", "dw", "decode"],
+    ap.add_argument("--only", choices=["quantize", "transpose", "fwd", "dx", "dw", "decode", "adamw"],
                     help="profiling aid: run just this kernel of the step (or the batched "
                          "M=1 decode) --warmup + --steps times and print its time")
     args = ap.parse_args()
@@ -688,6 +753,7 @@ def main():
             "quantize_48_layers_g128": quantize_sweep(tq, 5, 2),
             "out_proj_step": out_proj_step(tq, 200, 10),
             "sweep_48_layers": g_sweep(tq),
+            "adamw_requantize_g128": adamw_sweep(tq, 5, 2),
             "cublas_bf16_fwd_shape": cublas_context(tq),
             "hbm_peak_gbs": pk["hbm_gbs"],
         }

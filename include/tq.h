@@ -108,6 +108,38 @@ typedef struct {
 TQ_API tq_status tq_quantize_batched(const tq_quant_desc* descs, int32_t count, int32_t g,
                                      void* stream);
 
+/* Hyperparameters of one AdamW step (tq_adamw_requantize). */
+typedef struct tq_adamw_hparams {
+  double lr;            /* learning rate of this step (after any schedule), >= 0       */
+  double beta1, beta2;  /* in [0, 1); the paper uses (0.9, 0.95)                       */
+  double eps;           /* > 0; the paper gives none, the usual default is 1e-8         */
+  double weight_decay;  /* decoupled, >= 0; the paper uses 0.01                        */
+  double grad_scale;    /* multiplies the gradient, >= 0 (global-norm clip factor; 1)  */
+  int64_t step;         /* t >= 1: this update is the t-th of the moments              */
+} tq_adamw_hparams;
+
+/*
+ * tq_adamw_requantize — the optimizer step of §3.3 (AdamW on the fp32 latent
+ * weights, the training-hyperparameter table of the appendix) fused with the
+ * requantization of §3.1 (per-group absmean scale, ternary codes), in one pass:
+ *   g' = grad_scale * grad
+ *   m  = beta1 m + (1 - beta1) g'          v = beta2 v + (1 - beta2) g'^2
+ *   w  = w (1 - lr wd) - lr / (1 - beta1^t) * m / (sqrt(v) / sqrt(1 - beta2^t) + eps)
+ *   then codes / scales / zero_counts of the new w exactly as tq_quantize.
+ * Each operation is one fp32 operation in the order written (no fused
+ * multiply-add); the step constants are computed in fp64 and rounded once to
+ * fp32, so results are reproducible bit for bit.
+ *   w, m, v      in/out: fp32 [n][k], updated in place (device, 16-byte aligned).
+ *   grad         fp32 [n][k] (device).
+ *   codes, scales, zero_counts   out: as tq_quantize, for the updated w.
+ *   Requires the tq_quantize conditions on n, k, g; hp non-NULL with the ranges
+ *   above; TQ_ERR_INVALID_ARG otherwise, before anything is launched.
+ */
+TQ_API tq_status tq_adamw_requantize(float* w, const float* grad, float* m, float* v, int64_t n,
+                                     int64_t k, int32_t g, const tq_adamw_hparams* hp,
+                                     uint32_t* codes, float* scales, int32_t* zero_counts,
+                                     void* stream);
+
 /*
  * tq_linear_fwd — W1.58A16 forward (§3.1, "W1.58A16" of the title):
  *   y[m][n] = sum_k x[m][k] * s[n][k/g] * code[n][k].

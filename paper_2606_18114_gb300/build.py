@@ -18,7 +18,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OBJDIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libtq.so")
-SOURCES = ["tq_api.cu", "quantize.cu", "ts_gemm.cu", "dw_gemm.cu", "decode.cu"]
+SOURCES = ["tq_api.cu", "quantize.cu", "ts_gemm.cu", "dw_gemm.cu", "decode.cu", "adamw.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + [
     "-O3", "-lineinfo", "-std=c++17", "--expt-relaxed-constexpr",

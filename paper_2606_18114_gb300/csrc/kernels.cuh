@@ -56,6 +56,33 @@ cudaError_t launch_quantize_batched(QuantBatch<kQuantMaxMats>& batch, int g, int
 cudaError_t launch_transpose_codes(const uint32_t* codes, int64_t n, int64_t k, uint32_t* codes_t,
                                    cudaStream_t stream);
 
+// adamw.cu -------------------------------------------------------------------
+// Fused AdamW step + requantize of one weight matrix (flat, n * k weights).
+struct AdamwConst {     // fp32 step constants (computed in fp64 on the host)
+  float b1, omb1;       // beta1, 1 - beta1
+  float b2, omb2;       // beta2, 1 - beta2
+  float decay;          // 1 - lr * weight_decay
+  float step_size;      // lr / (1 - beta1^t)
+  float inv_bc2_sqrt;   // 1 / sqrt(1 - beta2^t)
+  float eps;
+  float grad_scale;     // multiplies the gradient (gradient clipping)
+};
+
+struct AdamwArgs {
+  float* w;             // fp32 [n][k], updated in place
+  const float* grad;    // fp32 [n][k]
+  float* m;             // fp32 [n][k], updated in place
+  float* v;             // fp32 [n][k], updated in place
+  uint32_t* codes;      // uint32 [n][k/16] of the new w
+  float* scales;        // fp32 [n][k/g]
+  int32_t* zeros;       // int32 [n][k/g]
+  int64_t total;        // n * k
+  AdamwConst c;
+};
+
+cudaError_t launch_adamw_requantize(const AdamwArgs& a, int g, int* status, int num_sms,
+                                    cudaStream_t stream);
+
 // ts_gemm.cu -----------------------------------------------------------------
 // Ternary x bf16 products with the expanded ternary weights as the tensor-memory
 // A operand. kTsFwd: out[m][n] = sum_k x[m][k] w^[n][k] (B = x, rows = n).

@@ -22,19 +22,13 @@
 // zero count of a word is 16 - popc(word & 0x5555...) because every non-zero code
 // has its low bit set).
 //
-// Code decision. The code is +-1 iff fl32(|w| / s) > 0.5 (round half to even sends
-// 0.5 to 0; the clip maps everything beyond 1.5 to +-1). The fp32 quotient exceeds
-// 0.5 exactly when the real quotient exceeds the midpoint 0.5 + 2^-25 between 0.5
-// and its successor, i.e. when |w| > s (1/2 + 2^-25). For a normal s that
-// threshold lies strictly between s/2 and the next fp32 value above s/2, so on
-// fp32 inputs the test is |w| > s/2 — one comparison reproduces the correctly
-// rounded division bit for bit (s/2 is exact for s >= 2^-125). Scales below
-// 2^-100 take the division.
+// Code decision: see quant_code.cuh.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
 #include "kernels.cuh"
 #include "ptx.cuh"
+#include "quant_code.cuh"
 
 namespace tq {
 namespace {
@@ -47,40 +41,6 @@ constexpr int kStageBytes = kStageW * 4;        // 32 KB
 constexpr int kStages = 3;                      // per CTA; two CTAs per SM
 constexpr int kCtasPerSm = 2;
 constexpr int kSmemBytes = kStages * kStageBytes + 2 * kStages * 8 + 128;
-
-// w |= bit when a > h (one compare and one predicated OR).
-__device__ __forceinline__ void or_if_gt(uint32_t& w, float a, float h, uint32_t bit) {
-  asm("{\n\t.reg .pred p;\n\tsetp.gt.f32 p, %1, %2;\n\t@p or.b32 %0, %0, %3;\n\t}"
-      : "+r"(w)
-      : "f"(a), "f"(h), "r"(bit));
-}
-
-// Code word of 16 consecutive weights; code j at bit p_j = 16*(j&1) + 2*(j>>1),
-// high bit the sign, low bit "non-zero".
-//   nz:  bit p_j set iff |w_j| > s/2 (fast path) or fl(|w_j| / s) > 0.5.
-//   neg: bit p_j + 1 set iff w_j < 0 (sign bit), for every j. The sign bits of
-//        weights 2i and 2i+1 (bound for bits 2i+1 and 2i+17) are gathered by one
-//        byte permute (bits 15 and 31), one shift and one masked OR.
-//   word = nz | (neg & (nz << 1)): the sign only where the code is non-zero.
-template <bool kDivide>
-__device__ __forceinline__ uint32_t code_word(const float (&x)[16], float s) {
-  uint32_t nz = 0, neg = 0;
-  if (kDivide) {
-#pragma unroll
-    for (int j = 0; j < 16; ++j)
-      or_if_gt(nz, fabsf(__fdiv_rn(x[j], s)), 0.5f, 1u << (16 * (j & 1) + 2 * (j >> 1)));
-  } else {
-    const float h = 0.5f * s;
-#pragma unroll
-    for (int j = 0; j < 16; ++j) or_if_gt(nz, fabsf(x[j]), h, 1u << (16 * (j & 1) + 2 * (j >> 1)));
-  }
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const uint32_t hi = __byte_perm(__float_as_uint(x[2 * i]), __float_as_uint(x[2 * i + 1]), 0x7632);
-    neg |= (hi >> (14 - 2 * i)) & ((1u << (2 * i + 1)) | (1u << (2 * i + 17)));
-  }
-  return nz | (neg & (nz << 1));
-}
 
 // Stage scheduler of one launch: {next dynamic stage, CTAs done}. Zero at the
 // start of a launch; the last CTA to finish claiming puts both back to zero.

@@ -6,6 +6,7 @@
 // stream.
 #include <cuda.h>
 #include <cuda_runtime.h>
+#include <math.h>
 #include <stdarg.h>
 #include <stdint.h>
 #include <stdio.h>
@@ -362,6 +363,50 @@ TQ_API tq_status tq_quantize_batched(const tq_quant_desc* descs, int32_t count, 
   cudaError_t e = tq::launch_quantize_batched(b, g, dev->status, dev->num_sms,
                                               static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? TQ_OK : cuda_fail(e, "quantize launch");
+}
+
+TQ_API tq_status tq_adamw_requantize(float* w, const float* grad, float* m, float* v, int64_t n,
+                                     int64_t k, int32_t g, const tq_adamw_hparams* hp,
+                                     uint32_t* codes, float* scales, int32_t* zero_counts,
+                                     void* stream) {
+  g_err[0] = 0;
+  TQ_TRY(check_quantize_args(w, n, k, g, codes, scales, zero_counts));
+  if (hp == nullptr) return fail(TQ_ERR_INVALID_ARG, "hparams is NULL");
+  if (hp->step < 1) return fail(TQ_ERR_INVALID_ARG, "step %lld < 1", (long long)hp->step);
+  const double lr = hp->lr, b1 = hp->beta1, b2 = hp->beta2, eps = hp->eps;
+  const double wd = hp->weight_decay, gs = hp->grad_scale;
+  if (!(lr >= 0 && lr < 1e30) || !(b1 >= 0 && b1 < 1) || !(b2 >= 0 && b2 < 1) ||
+      !(eps > 0 && eps < 1e30) || !(wd >= 0 && wd < 1e30) || !(gs >= 0 && gs < 1e30))
+    return fail(TQ_ERR_INVALID_ARG, "hyperparameters out of range");
+  if (n == 0 || k == 0) return TQ_OK;
+  TQ_TRY(check_ptr(grad, "grad"));
+  TQ_TRY(check_ptr(m, "m"));
+  TQ_TRY(check_ptr(v, "v"));
+  tq::AdamwArgs a{};
+  a.w = w;
+  a.grad = grad;
+  a.m = m;
+  a.v = v;
+  a.codes = codes;
+  a.scales = scales;
+  a.zeros = zero_counts;
+  a.total = n * k;
+  // step constants: fp64, rounded once to fp32
+  const double t = static_cast<double>(hp->step);
+  a.c.b1 = static_cast<float>(b1);
+  a.c.omb1 = static_cast<float>(1.0 - b1);
+  a.c.b2 = static_cast<float>(b2);
+  a.c.omb2 = static_cast<float>(1.0 - b2);
+  a.c.decay = static_cast<float>(1.0 - lr * wd);
+  a.c.step_size = static_cast<float>(lr / (1.0 - pow(b1, t)));
+  a.c.inv_bc2_sqrt = static_cast<float>(1.0 / sqrt(1.0 - pow(b2, t)));
+  a.c.eps = static_cast<float>(eps);
+  a.c.grad_scale = static_cast<float>(gs);
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaError_t e = tq::launch_adamw_requantize(a, g, dev->status, dev->num_sms,
+                                              static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "adamw launch");
 }
 
 TQ_API tq_status tq_linear_fwd(const void* x, int64_t m, int64_t k, const uint32_t* codes,

@@ -25,6 +25,8 @@ __all__ = [
     "linear_fwd_batched",
     "fwd_batch",
     "device_status",
+    "adamw_requantize",
+    "AdamwHparams",
     "version",
     "OUT_F32",
     "OUT_BF16",
@@ -38,7 +40,7 @@ STATUS = {0: "TQ_OK", 1: "TQ_ERR_INVALID_ARG", 2: "TQ_ERR_UNSUPPORTED", 3: "TQ_E
 # Every symbol include/tq.h declares.
 EXPORTS = ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
            "tq_linear_bwd_noalloc", "tq_codes_transpose", "tq_linear_fwd_batched",
-           "tq_device_status", "tq_last_error", "tq_version")
+           "tq_adamw_requantize", "tq_device_status", "tq_last_error", "tq_version")
 
 _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtq.so")
 _lib = None
@@ -58,6 +60,19 @@ class QuantDesc(ctypes.Structure):
         ("zero_counts", ctypes.c_void_p),
         ("n", ctypes.c_int64),
         ("k", ctypes.c_int64),
+    ]
+
+
+class AdamwHparams(ctypes.Structure):
+    """tq_adamw_hparams of include/tq.h."""
+    _fields_ = [
+        ("lr", ctypes.c_double),
+        ("beta1", ctypes.c_double),
+        ("beta2", ctypes.c_double),
+        ("eps", ctypes.c_double),
+        ("weight_decay", ctypes.c_double),
+        ("grad_scale", ctypes.c_double),
+        ("step", ctypes.c_int64),
     ]
 
 
@@ -93,6 +108,8 @@ def load(path: Optional[str] = None):
     lib.tq_codes_transpose.argtypes = [vp, i64, i64, vp, vp]
     lib.tq_linear_fwd_batched.argtypes = [ctypes.POINTER(FwdDesc), i32, i64, vp]
     lib.tq_device_status.argtypes = [vp]
+    lib.tq_adamw_requantize.argtypes = [vp, vp, vp, vp, i64, i64, i32, ctypes.POINTER(AdamwHparams),
+                                        vp, vp, vp, vp]
     for name in ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
                  "tq_linear_bwd_noalloc", "tq_codes_transpose", "tq_linear_fwd_batched",
                  "tq_device_status"):
@@ -149,6 +166,28 @@ def quantize(w: torch.Tensor, g: int, out=None, stream=None):
         codes, scales, zeros = out
     _check(load().tq_quantize(_ptr(w), n, k, g, _ptr(codes), _ptr(scales), _ptr(zeros),
                               _stream(stream)))
+    return codes, scales, zeros
+
+
+def adamw_requantize(w: torch.Tensor, grad: torch.Tensor, m: torch.Tensor, v: torch.Tensor,
+                     g: int, lr: float, step: int, beta1: float = 0.9, beta2: float = 0.95,
+                     eps: float = 1e-8, weight_decay: float = 0.01, grad_scale: float = 1.0,
+                     out=None, stream=None):
+    """One AdamW step on the fp32 latent ``w`` (``m``, ``v`` its moments; all three
+    updated in place) fused with the requantization of the new weights.
+
+    Returns ``(codes, scales, zero_counts)`` as :func:`quantize` does."""
+    n, k = w.shape
+    if out is None:
+        codes = torch.empty((n, k // 16), dtype=torch.int32, device=w.device)
+        scales = torch.empty((n, k // g), dtype=torch.float32, device=w.device)
+        zeros = torch.empty((n, k // g), dtype=torch.int32, device=w.device)
+    else:
+        codes, scales, zeros = out
+    hp = AdamwHparams(lr, beta1, beta2, eps, weight_decay, grad_scale, step)
+    _check(load().tq_adamw_requantize(_ptr(w), _ptr(grad), _ptr(m), _ptr(v), n, k, g,
+                                      ctypes.byref(hp), _ptr(codes), _ptr(scales), _ptr(zeros),
+                                      _stream(stream)))
     return codes, scales, zeros
 
 

@@ -147,3 +147,27 @@ def test_quantize_batched_rejects_before_launch(lib):
     assert lib.tq_quantize_batched(arr, -1, 64, None) == 1    # negative count
     assert lib.tq_quantize_batched(None, 2, 64, None) == 1    # null descs
     assert lib.tq_quantize_batched(None, 0, 64, None) == 0    # nothing to do
+
+
+def test_adamw_requantize_rejects_before_launch(lib):
+    """Every argument error is reported before anything touches the device."""
+    from paper_2606_18114_gb300.tq import AdamwHparams
+    import ctypes
+    good = AdamwHparams(2.5e-4, 0.9, 0.95, 1e-8, 0.01, 1.0, 1)
+    hp = ctypes.byref(good)
+    f = lib.tq_adamw_requantize
+    assert f(FAKE, FAKE, FAKE, FAKE, 8, 256, 128, None, FAKE, FAKE, FAKE, None) == 1  # no hparams
+    assert b"hparams" in lib.tq_last_error()
+    for bad in (AdamwHparams(2.5e-4, 0.9, 0.95, 1e-8, 0.01, 1.0, 0),    # step 0
+                AdamwHparams(2.5e-4, 1.0, 0.95, 1e-8, 0.01, 1.0, 1),    # beta1 = 1
+                AdamwHparams(2.5e-4, 0.9, -0.1, 1e-8, 0.01, 1.0, 1),    # beta2 < 0
+                AdamwHparams(-1e-3, 0.9, 0.95, 1e-8, 0.01, 1.0, 1),     # lr < 0
+                AdamwHparams(2.5e-4, 0.9, 0.95, 0.0, 0.01, 1.0, 1),     # eps = 0
+                AdamwHparams(2.5e-4, 0.9, 0.95, 1e-8, 0.01, float("nan"), 1)):
+        assert f(FAKE, FAKE, FAKE, FAKE, 8, 256, 128, ctypes.byref(bad), FAKE, FAKE, FAKE, None) == 1
+    assert f(FAKE, FAKE, FAKE, FAKE, 8, 96, 64, hp, FAKE, FAKE, FAKE, None) == 1     # k % g
+    assert f(FAKE, FAKE, FAKE, FAKE, 8, 256, 48, hp, FAKE, FAKE, FAKE, None) == 1    # group size
+    assert f(FAKE, MIS, FAKE, FAKE, 8, 256, 128, hp, FAKE, FAKE, FAKE, None) == 1    # misaligned grad
+    assert b"grad" in lib.tq_last_error()
+    assert f(FAKE, FAKE, None, FAKE, 8, 256, 128, hp, FAKE, FAKE, FAKE, None) == 1   # null m
+    assert f(FAKE, FAKE, FAKE, FAKE, 0, 256, 128, hp, FAKE, FAKE, FAKE, None) == 0   # empty: nothing
