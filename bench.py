@@ -514,6 +514,47 @@ def adamw_sweep(tq, steps, warmup):
     return res
 
 
+def decoupled_sweep(tq, steps, warmup):
+    """The decoupled quantizer on in_proj with the asymmetric gate (rows 0..4095 at
+    0.8 x absmean), and the magnitude gradient dalpha = sum dW * c per group."""
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(41)
+    pk, _ = peaks()
+    n, k = IN_PROJ
+    w = torch.randn((n, k), generator=gen, device="cuda") * 0.02
+    dw = torch.randn((n, k), generator=gen, device="cuda")
+    f = torch.ones(n, device="cuda")
+    f[:4096] = 0.8
+    out = (torch.empty((n, k // 16), dtype=torch.int32, device="cuda"),
+           torch.empty((n, k // G), device="cuda"),
+           torch.empty((n, k // G), dtype=torch.int32, device="cuda"))
+    da = torch.empty((n, k // G), device="cuda")
+    res = {}
+    for label, fn, nbytes in (
+            ("quantize_decoupled", lambda: tq.quantize_decoupled(w, G, f, out=out),
+             n * k * 4 + n * k // 4 + 8 * n * k // G + 4 * n),
+            ("alpha_grad", lambda: tq.alpha_grad(dw, out[0], G, out=da),
+             n * k * 4 + n * k // 4 + 4 * n * k // G)):
+        for _ in range(warmup):
+            fn()
+        torch.cuda.synchronize()
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record()
+        for _ in range(steps):
+            fn()
+        t1.record()
+        torch.cuda.synchronize()
+        ms = t0.elapsed_time(t1) / steps
+        res[label] = {"us": round(ms * 1e3, 2), "GB/s": round(nbytes / ms / 1e6, 1),
+                      "frac": round(nbytes / ms / 1e6 / pk["hbm_gbs"], 4), "bytes": nbytes}
+    zr = out[2].double()
+    res["zero_ratio_gate_rows"] = round(float(zr[:4096].mean()) / G, 4)
+    res["zero_ratio_other_rows"] = round(float(zr[4096:].mean()) / G, 4)
+    tq.device_status()
+    return res
+
+
 def cublas_context(tq):
     """cuBLAS bf16 dense GEMM of the forward's shape (Y = X W^T, 16384 x 8512 x 2048):
     context for the tensor-core fraction, not part of the path."""
@@ -754,6 +795,7 @@ def main():
             "out_proj_step": out_proj_step(tq, 200, 10),
             "sweep_48_layers": g_sweep(tq),
             "adamw_requantize_g128": adamw_sweep(tq, 5, 2),
+            "decoupled_in_proj": decoupled_sweep(tq, 20, 3),
             "cublas_bf16_fwd_shape": cublas_context(tq),
             "hbm_peak_gbs": pk["hbm_gbs"],
         }

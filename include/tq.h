@@ -108,6 +108,36 @@ typedef struct {
 TQ_API tq_status tq_quantize_batched(const tq_quant_desc* descs, int32_t count, int32_t g,
                                      void* stream);
 
+/*
+ * tq_quantize_decoupled — the decoupled quantizer of the paper's decoupled-
+ * quantization ablation (appendix): the codes are decided against a threshold
+ *   tau_g = row_factor[n] * s_g   (one fp32 product; s_g the absmean of §3.1)
+ * instead of s_g itself, so that sparsity (tau) and output magnitude (a separate
+ * learnable alpha_g the caller keeps and passes as the scales of tq_linear_fwd /
+ * tq_linear_bwd) are decoupled; the asymmetric-gate variant uses 0.8 on the gate
+ * rows 0..4095 of in_proj and 1 elsewhere.
+ *   row_factor   fp32 [n] on the device, or NULL (every factor 1: tq_quantize).
+ *   scales       out: the absmean s_g (not tau), e.g. to initialise alpha.
+ *   Other arguments, layouts and errors as tq_quantize.
+ */
+TQ_API tq_status tq_quantize_decoupled(const float* w, int64_t n, int64_t k, int32_t g,
+                                       const float* row_factor, uint32_t* codes, float* scales,
+                                       int32_t* zero_counts, void* stream);
+
+/*
+ * tq_alpha_grad — gradient of the decoupled quantizer's magnitude: with
+ * W^ = alpha_g * c, dalpha[n][j] = sum over group j of row n of dW^ * c, where dW^
+ * is the dW of tq_linear_bwd (the STE hands the same matrix to the latent W).
+ *   dw       fp32 [n][k] (device, 16-byte aligned).
+ *   codes    uint32 [n][k/16], layout of tq_quantize (device, 16-byte aligned).
+ *   dalpha   out: fp32 [n][k/g] (device).
+ *   Summation: each 16-weight word in weight order, then the group's words as a
+ *   binary tree; fp32. Requires k % g == 0 (and so k % 16 == 0); TQ_ERR_INVALID_ARG
+ *   otherwise.
+ */
+TQ_API tq_status tq_alpha_grad(const float* dw, const uint32_t* codes, int64_t n, int64_t k,
+                               int32_t g, float* dalpha, void* stream);
+
 /* Hyperparameters of one AdamW step (tq_adamw_requantize). */
 typedef struct tq_adamw_hparams {
   double lr;            /* learning rate of this step (after any schedule), >= 0       */

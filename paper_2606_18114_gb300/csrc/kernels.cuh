@@ -25,9 +25,11 @@ cudaError_t ensure_smem_limit(int bytes) {
 }
 
 // quantize.cu ----------------------------------------------------------------
+// row_factor (fp32 [n] or null): the codes of row r are decided against the
+// threshold row_factor[r] * s instead of s (the decoupled quantizer); scales stay s.
 cudaError_t launch_quantize(const float* w, int64_t n, int64_t k, int g, uint32_t* codes,
                             float* scales, int32_t* zeros, int* status, int num_sms,
-                            cudaStream_t stream);
+                            cudaStream_t stream, const float* row_factor = nullptr);
 
 // Many matrices (same group size) in one launch.
 struct QuantMat {
@@ -37,7 +39,14 @@ struct QuantMat {
   int32_t* zeros;   // int32 [n][k/g]
   int64_t total;    // n * k
   int64_t stage0;   // first stage of this matrix (set by the launcher)
+  const float* row_factor;  // null, or fp32 [n]: per-row threshold factor
+  int64_t k;        // row length (for row_factor)
 };
+
+// dalpha[n][k/g] = sum over each group of dw * code (the decoupled quantizer's
+// magnitude gradient).
+cudaError_t launch_alpha_grad(const float* dw, const uint32_t* codes, int64_t n, int64_t k, int g,
+                              float* dalpha, int num_sms, cudaStream_t stream);
 
 template <int kMax>
 struct QuantBatch {

@@ -183,13 +183,15 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 #pragma unroll
       for (int off = 1; off < kLanesPerGroup; off <<= 1) sum += __shfl_xor_sync(live, sum, off);
       const float s = sum * kInvG;  // s = (1/g) * sum |w|
+      // the decoupled quantizer decides against tau = f_row * s (one fp32 product)
+      const float tau = mt.row_factor == nullptr ? s : __fmul_rn(s, mt.row_factor[e / mt.k]);
       const float x[16] = {v[0].x, v[0].y, v[0].z, v[0].w, v[1].x, v[1].y, v[1].z, v[1].w,
                            v[2].x, v[2].y, v[2].z, v[2].w, v[3].x, v[3].y, v[3].z, v[3].w};
-      // scales below 2^-100 (all-zero or denormal groups) take the division
-      const bool tiny = s < 0x1p-100f;
+      // thresholds below 2^-100 (all-zero or denormal groups) take the division
+      const bool tiny = tau < 0x1p-100f;
       const uint32_t word = __any_sync(live, tiny)
-                                ? (tiny ? code_word<true>(x, s) : code_word<false>(x, s))
-                                : code_word<false>(x, s);
+                                ? (tiny ? code_word<true>(x, tau) : code_word<false>(x, tau))
+                                : code_word<false>(x, tau);
       const unsigned gmask =
           kLanesPerGroup == 32 ? 0xffffffffu
                                : ((1u << kLanesPerGroup) - 1u) << (lane & ~(kLanesPerGroup - 1));
@@ -292,6 +294,74 @@ __global__ void __launch_bounds__(256) transpose_codes_kernel(const uint32_t* __
 
 }  // namespace
 
+namespace {
+
+// Magnitude gradient of the decoupled quantizer: dalpha_g = sum over the group of
+// dW * c. A lane takes one code word (16 weights, its dW as four float4) and adds
+// the dW of its non-zero codes with their signs, in weight order; the g/16 lanes
+// of a group then add their sums with xor-shuffles (groups lie within one warp's
+// 32 words, and a warp holds whole groups). Plain vector loads: a secondary pass.
+template <int G>
+__global__ void __launch_bounds__(256) alpha_grad_kernel(const float* __restrict__ dw,
+                                                         const uint32_t* __restrict__ codes,
+                                                         int64_t words, float* __restrict__ dalpha) {
+  constexpr int kLanesPerGroup = G / 16;
+  const int lane = threadIdx.x & 31;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
+       base < words; base += stride) {
+    const int64_t wi = base + lane;
+    if (wi >= words) continue;  // whole groups: the lanes of a group agree
+    const uint32_t c = __ldg(codes + wi);
+    const float4* p = reinterpret_cast<const float4*>(dw + wi * 16);
+    float sum = 0.f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 v4 = __ldg(p + q);
+      const float v[4] = {v4.x, v4.y, v4.z, v4.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int j = 4 * q + i;
+        const int bit = 16 * (j & 1) + 2 * (j >> 1);  // code j of the word (include/tq.h)
+        const float t = (c >> (bit + 1)) & 1u ? -v[i] : v[i];
+        sum += (c >> bit) & 1u ? t : 0.f;
+      }
+    }
+    const unsigned gmask =
+        kLanesPerGroup == 32 ? 0xffffffffu
+                             : ((1u << kLanesPerGroup) - 1u) << (lane & ~(kLanesPerGroup - 1));
+#pragma unroll
+    for (int off = 1; off < kLanesPerGroup; off <<= 1) sum += __shfl_xor_sync(gmask, sum, off);
+    if ((lane & (kLanesPerGroup - 1)) == 0) dalpha[wi / kLanesPerGroup] = sum;
+  }
+}
+
+template <int G>
+cudaError_t launch_ag(const float* dw, const uint32_t* codes, int64_t words, float* dalpha,
+                      int num_sms, cudaStream_t stream) {
+  const int64_t need = (words + 255) / 256;
+  const int64_t cap = static_cast<int64_t>(num_sms) * 8;
+  alpha_grad_kernel<G><<<static_cast<unsigned>(need < cap ? need : cap), 256, 0, stream>>>(
+      dw, codes, words, dalpha);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_alpha_grad(const float* dw, const uint32_t* codes, int64_t n, int64_t k, int g,
+                              float* dalpha, int num_sms, cudaStream_t stream) {
+  const int64_t words = n * k / 16;
+  if (words <= 0) return cudaSuccess;
+  switch (g) {
+    case 32: return launch_ag<32>(dw, codes, words, dalpha, num_sms, stream);
+    case 64: return launch_ag<64>(dw, codes, words, dalpha, num_sms, stream);
+    case 128: return launch_ag<128>(dw, codes, words, dalpha, num_sms, stream);
+    case 256: return launch_ag<256>(dw, codes, words, dalpha, num_sms, stream);
+    case 512: return launch_ag<512>(dw, codes, words, dalpha, num_sms, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 cudaError_t launch_transpose_codes(const uint32_t* codes, int64_t n, int64_t k, uint32_t* codes_t,
                                    cudaStream_t stream) {
   const int64_t ldt = 4 * ((n + 63) / 64);
@@ -302,9 +372,9 @@ cudaError_t launch_transpose_codes(const uint32_t* codes, int64_t n, int64_t k, 
 
 cudaError_t launch_quantize(const float* w, int64_t n, int64_t k, int g, uint32_t* codes,
                             float* scales, int32_t* zeros, int* status, int num_sms,
-                            cudaStream_t stream) {
+                            cudaStream_t stream, const float* row_factor) {
   QuantBatch<1> b{};
-  b.mats[0] = QuantMat{w, codes, scales, zeros, n * k, 0};
+  b.mats[0] = QuantMat{w, codes, scales, zeros, n * k, 0, row_factor, k};
   b.count = 1;
   b.nstages = (n * k + kStageW - 1) / kStageW;
   return launch_g<1>(b, g, status, num_sms, stream);

@@ -337,6 +337,40 @@ TQ_API tq_status tq_quantize(const float* w, int64_t n, int64_t k, int32_t g, ui
   return e == cudaSuccess ? TQ_OK : cuda_fail(e, "quantize launch");
 }
 
+TQ_API tq_status tq_quantize_decoupled(const float* w, int64_t n, int64_t k, int32_t g,
+                                       const float* row_factor, uint32_t* codes, float* scales,
+                                       int32_t* zero_counts, void* stream) {
+  g_err[0] = 0;
+  TQ_TRY(check_quantize_args(w, n, k, g, codes, scales, zero_counts));
+  if (n == 0 || k == 0) return TQ_OK;
+  if (row_factor != nullptr && (reinterpret_cast<uintptr_t>(row_factor) & 3) != 0)
+    return fail(TQ_ERR_INVALID_ARG, "row_factor is not 4-byte aligned");
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaError_t e = tq::launch_quantize(w, n, k, g, codes, scales, zero_counts, dev->status,
+                                      dev->num_sms, static_cast<cudaStream_t>(stream), row_factor);
+  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "quantize launch");
+}
+
+TQ_API tq_status tq_alpha_grad(const float* dw, const uint32_t* codes, int64_t n, int64_t k,
+                               int32_t g, float* dalpha, void* stream) {
+  g_err[0] = 0;
+  if (n < 0 || k < 0) return fail(TQ_ERR_INVALID_ARG, "negative size");
+  if (log2_group(g) < 0) return fail(TQ_ERR_INVALID_ARG, "group size %d not in {32..512}", g);
+  if (k % g != 0) return fail(TQ_ERR_INVALID_ARG, "k=%lld is not a multiple of g=%d", (long long)k, g);
+  if (n == 0 || k == 0) return TQ_OK;
+  if (n > INT64_MAX / k) return fail(TQ_ERR_INVALID_ARG, "n*k overflows");
+  TQ_TRY(check_ptr(dw, "dw"));
+  TQ_TRY(check_ptr(codes, "codes"));
+  if (dalpha == nullptr || (reinterpret_cast<uintptr_t>(dalpha) & 3) != 0)
+    return fail(TQ_ERR_INVALID_ARG, "dalpha is NULL or not 4-byte aligned");
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaError_t e = tq::launch_alpha_grad(dw, codes, n, k, g, dalpha, dev->num_sms,
+                                        static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "alpha_grad launch");
+}
+
 TQ_API tq_status tq_quantize_batched(const tq_quant_desc* descs, int32_t count, int32_t g,
                                      void* stream) {
   g_err[0] = 0;
@@ -355,7 +389,7 @@ TQ_API tq_status tq_quantize_batched(const tq_quant_desc* descs, int32_t count, 
       return fail(st, "descs[%d]: %s", i, msg);
     }
     if (d.n == 0 || d.k == 0) continue;
-    b.mats[b.count++] = tq::QuantMat{d.w, d.codes, d.scales, d.zero_counts, d.n * d.k, 0};
+    b.mats[b.count++] = tq::QuantMat{d.w, d.codes, d.scales, d.zero_counts, d.n * d.k, 0, nullptr, d.k};
   }
   if (b.count == 0) return TQ_OK;
   const DeviceInfo* dev = nullptr;

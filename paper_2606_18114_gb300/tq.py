@@ -26,6 +26,8 @@ __all__ = [
     "fwd_batch",
     "device_status",
     "adamw_requantize",
+    "quantize_decoupled",
+    "alpha_grad",
     "AdamwHparams",
     "version",
     "OUT_F32",
@@ -40,7 +42,8 @@ STATUS = {0: "TQ_OK", 1: "TQ_ERR_INVALID_ARG", 2: "TQ_ERR_UNSUPPORTED", 3: "TQ_E
 # Every symbol include/tq.h declares.
 EXPORTS = ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
            "tq_linear_bwd_noalloc", "tq_codes_transpose", "tq_linear_fwd_batched",
-           "tq_adamw_requantize", "tq_device_status", "tq_last_error", "tq_version")
+           "tq_adamw_requantize", "tq_quantize_decoupled", "tq_alpha_grad",
+           "tq_device_status", "tq_last_error", "tq_version")
 
 _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtq.so")
 _lib = None
@@ -108,6 +111,8 @@ def load(path: Optional[str] = None):
     lib.tq_codes_transpose.argtypes = [vp, i64, i64, vp, vp]
     lib.tq_linear_fwd_batched.argtypes = [ctypes.POINTER(FwdDesc), i32, i64, vp]
     lib.tq_device_status.argtypes = [vp]
+    lib.tq_quantize_decoupled.argtypes = [vp, i64, i64, i32, vp, vp, vp, vp, vp]
+    lib.tq_alpha_grad.argtypes = [vp, vp, i64, i64, i32, vp, vp]
     lib.tq_adamw_requantize.argtypes = [vp, vp, vp, vp, i64, i64, i32, ctypes.POINTER(AdamwHparams),
                                         vp, vp, vp, vp]
     for name in ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
@@ -189,6 +194,33 @@ def adamw_requantize(w: torch.Tensor, grad: torch.Tensor, m: torch.Tensor, v: to
                                       ctypes.byref(hp), _ptr(codes), _ptr(scales), _ptr(zeros),
                                       _stream(stream)))
     return codes, scales, zeros
+
+
+def quantize_decoupled(w: torch.Tensor, g: int, row_factor: Optional[torch.Tensor] = None,
+                       out=None, stream=None):
+    """The decoupled quantizer: codes against ``row_factor[n] * absmean`` (``None``: 1).
+    Returns ``(codes, absmean scales, zero_counts)`` like :func:`quantize`."""
+    n, k = w.shape
+    if out is None:
+        codes = torch.empty((n, k // 16), dtype=torch.int32, device=w.device)
+        scales = torch.empty((n, k // g), dtype=torch.float32, device=w.device)
+        zeros = torch.empty((n, k // g), dtype=torch.int32, device=w.device)
+    else:
+        codes, scales, zeros = out
+    rf = None if row_factor is None else _ptr(row_factor)
+    _check(load().tq_quantize_decoupled(_ptr(w), n, k, g, rf, _ptr(codes), _ptr(scales),
+                                        _ptr(zeros), _stream(stream)))
+    return codes, scales, zeros
+
+
+def alpha_grad(dw: torch.Tensor, codes: torch.Tensor, g: int, out: Optional[torch.Tensor] = None,
+               stream=None) -> torch.Tensor:
+    """Gradient of the decoupled quantizer's magnitude: per group, sum of dW * code."""
+    n, k = dw.shape
+    if out is None:
+        out = torch.empty((n, k // g), dtype=torch.float32, device=dw.device)
+    _check(load().tq_alpha_grad(_ptr(dw), _ptr(codes), n, k, g, _ptr(out), _stream(stream)))
+    return out
 
 
 def quant_batch(items: Sequence[tuple]):

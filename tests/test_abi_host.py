@@ -171,3 +171,19 @@ def test_adamw_requantize_rejects_before_launch(lib):
     assert b"grad" in lib.tq_last_error()
     assert f(FAKE, FAKE, None, FAKE, 8, 256, 128, hp, FAKE, FAKE, FAKE, None) == 1   # null m
     assert f(FAKE, FAKE, FAKE, FAKE, 0, 256, 128, hp, FAKE, FAKE, FAKE, None) == 0   # empty: nothing
+
+
+def test_decoupled_and_alpha_grad_reject_before_launch(lib):
+    q, ag = lib.tq_quantize_decoupled, lib.tq_alpha_grad
+    assert q(FAKE, 8, 96, 64, None, FAKE, FAKE, FAKE, None) == 1          # k % g
+    assert q(FAKE, 8, 256, 48, None, FAKE, FAKE, FAKE, None) == 1         # group size
+    assert q(MIS, 8, 256, 128, None, FAKE, FAKE, FAKE, None) == 1         # misaligned w
+    assert q(FAKE, 8, 256, 128, FAKE + 2, FAKE, FAKE, FAKE, None) == 1    # misaligned factors
+    assert b"row_factor" in lib.tq_last_error()
+    assert q(FAKE, 0, 256, 128, None, FAKE, FAKE, FAKE, None) == 0        # empty
+    assert ag(FAKE, FAKE, 8, 96, 64, FAKE, None) == 1                     # k % g
+    assert ag(FAKE, FAKE, 8, 256, 16, FAKE, None) == 1                    # group size
+    assert ag(MIS, FAKE, 8, 256, 128, FAKE, None) == 1                    # misaligned dw
+    assert ag(FAKE, FAKE, 8, 256, 128, None, None) == 1                   # null dalpha
+    assert ag(FAKE, FAKE, -1, 256, 128, FAKE, None) == 1                  # negative size
+    assert ag(FAKE, FAKE, 0, 256, 128, FAKE, None) == 0                   # empty
