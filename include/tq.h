@@ -64,7 +64,12 @@ typedef enum {
 
 typedef enum {
   TQ_OUT_F32 = 0,  /* fp32 output (default: keeps the max-element error small) */
-  TQ_OUT_BF16 = 1  /* bf16 output, round to nearest even                        */
+  TQ_OUT_BF16 = 1, /* bf16 output, round to nearest even                        */
+  /* Flag OR-ed into an output type (y_dtype, dx_dtype, tq_fwd_desc.y_dtype): the
+   * activations x and dy are fp16 instead of bf16 (the paper's A16 is FP16, §3.3).
+   * The codes expand to the same +-1 values; the group scale is rounded to fp16
+   * instead of bf16 where the kernels apply it to the expanded codes. */
+  TQ_IN_F16 = 0x100
 } tq_out_dtype;
 
 /*
@@ -175,7 +180,8 @@ TQ_API tq_status tq_adamw_requantize(float* w, const float* grad, float* m, floa
  *   y[m][n] = sum_k x[m][k] * s[n][k/g] * code[n][k].
  *   x            bf16 [m][k] activations.
  *   codes/scales as produced by tq_quantize for W [n][k].
- *   y            out: [m][n], fp32 (TQ_OUT_F32) or bf16 (TQ_OUT_BF16).
+ *   y            out: [m][n], fp32 (TQ_OUT_F32) or bf16 (TQ_OUT_BF16); y_dtype may
+ *                carry TQ_IN_F16 (x is fp16).
  *   Requires k % 64 == 0 and k % g == 0; n >= 1 when m >= 1.
  *   m <= 16 runs the decode kernel, larger m the tensor-core GEMM; both expand
  *   the codes on chip and accumulate in fp32 (the decode kernel folds the fp32

@@ -49,6 +49,7 @@
 // segments need range guards); per segment it runs one wait, its chunks and one
 // arrival.
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -124,9 +125,14 @@ struct SegInfo {
 };
 static_assert(sizeof(SegInfo) == 48, "segment descriptor");
 
+// Two 16-bit products in the activation type (bf16, or fp16 with F16).
+template <bool F16>
 __device__ __forceinline__ uint32_t bmul2(uint32_t a, uint32_t b) {
   uint32_t d;
-  asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  if constexpr (F16)
+    asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  else
+    asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
   return d;
 }
 
@@ -147,26 +153,42 @@ __device__ __forceinline__ uint32_t opaque(uint32_t v) {
   return r;
 }
 
+// mma.sync m16n8k16, A and B in the activation type (both bf16, or both fp16).
+template <bool F16>
 __device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                          uint32_t a3, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
-      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+  if constexpr (F16)
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, "
+        "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+  else
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+        "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// The same with a zero accumulator input (the first product of a group).
+// The same with a zero accumulator input.
+template <bool F16>
 __device__ __forceinline__ void mma16816_zc(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                             uint32_t a3, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
-      "{%4, %5, %6, %7}, {%8, %9}, {%10, %10, %10, %10};"
-      : "=f"(c[0]), "=f"(c[1]), "=f"(c[2]), "=f"(c[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(0.0f));
+  if constexpr (F16)
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, "
+        "{%4, %5, %6, %7}, {%8, %9}, {%10, %10, %10, %10};"
+        : "=f"(c[0]), "=f"(c[1]), "=f"(c[2]), "=f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(0.0f));
+  else
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+        "{%4, %5, %6, %7}, {%8, %9}, {%10, %10, %10, %10};"
+        : "=f"(c[0]), "=f"(c[1]), "=f"(c[2]), "=f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(0.0f));
 }
 
-// 16-byte global -> shared copy (L2 only); zero-filled when src_bytes is 0.
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
                "r"(src_bytes)
@@ -185,9 +207,14 @@ __device__ __forceinline__ void cp_async_arrive(uint32_t bar) {
   asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
 }
 
-__device__ __forceinline__ uint32_t half_scale_bf16x2(float s) {
-  const __nv_bfloat16 h = __float2bfloat16_rn(0.5f * s);
-  const uint32_t u = __bfloat16_as_ushort(h);
+// s / 2 rounded to the activation type, in both halves.
+template <bool F16>
+__device__ __forceinline__ uint32_t half_scale_x2(float s) {
+  uint32_t u;
+  if constexpr (F16)
+    u = __half_as_ushort(__float2half_rn(0.5f * s));
+  else
+    u = __bfloat16_as_ushort(__float2bfloat16_rn(0.5f * s));
   return u | (u << 16);
 }
 
@@ -207,7 +234,7 @@ __device__ __forceinline__ int find_mat(const DecodeBatch& b, int u) {
 constexpr int kSchedSlots = 256;
 __device__ uint32_t g_dsched[kSchedSlots][2];
 
-template <bool kTwoTiles>
+template <bool kTwoTiles, bool F16>
 __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     decode_kernel(const __grid_constant__ DecodeBatch b, uint32_t* sched) {
   constexpr int kConsumers = DecodeCfg<kTwoTiles>::kConsumers;
@@ -317,7 +344,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
         __syncwarp();
         if (lane < m)
           bulk_load(xdst + lane * kXTokBytes,
-                    static_cast<const __nv_bfloat16*>(mt.x) + lane * mt.k +
+                    static_cast<const uint16_t*>(mt.x) + lane * mt.k +
                         static_cast<int64_t>(s) * kSegK,
                     xbytes, full_bar(slot), keep_policy);
         if (mt.scale_mode == kDecodeScaleUnit) {
@@ -541,11 +568,11 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
               const uint32_t a2 = pair_bits(u0, j + 1, mul[j + 1]);
               const uint32_t a3 = pair_bits(u1, j + 1, mul[j + 1]);
               if (kb == 0) {
-                mma16816_zc(p[r], a0, a1, a2, a3, xr[0], xr[1]);
-                if (kTwoTiles) mma16816_zc(p1[r], a0, a1, a2, a3, yr[0], yr[1]);
+                mma16816_zc<F16>(p[r], a0, a1, a2, a3, xr[0], xr[1]);
+                if (kTwoTiles) mma16816_zc<F16>(p1[r], a0, a1, a2, a3, yr[0], yr[1]);
               } else {
-                mma16816(p[r], a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
-                if (kTwoTiles) mma16816(p1[r], a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
+                mma16816<F16>(p[r], a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
+                if (kTwoTiles) mma16816<F16>(p1[r], a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
               }
             }
           }
@@ -569,22 +596,22 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
           const int qa = (kc + 16 * t) >> log2g, qb = (kc + 64 + 16 * t) >> log2g;
 #pragma unroll
           for (int r = 0; r < kTiles; ++r) {
-            const uint32_t hs0a = half_scale_bf16x2(sl[soff[r][0] + qa]);
-            const uint32_t hs1a = half_scale_bf16x2(sl[soff[r][1] + qa]);
-            const uint32_t hs0b = khi ? half_scale_bf16x2(sl[soff[r][0] + qb]) : 0u;
-            const uint32_t hs1b = khi ? half_scale_bf16x2(sl[soff[r][1] + qb]) : 0u;
+            const uint32_t hs0a = half_scale_x2<F16>(sl[soff[r][0] + qa]);
+            const uint32_t hs1a = half_scale_x2<F16>(sl[soff[r][1] + qa]);
+            const uint32_t hs0b = khi ? half_scale_x2<F16>(sl[soff[r][0] + qb]) : 0u;
+            const uint32_t hs1b = khi ? half_scale_x2<F16>(sl[soff[r][1] + qb]) : 0u;
 #pragma unroll
             for (int kb = 0; kb < 8; ++kb) {
               const int j = 2 * (kb & 3);
               const uint32_t u0 = kb < 4 ? w[r][0].x : w[r][0].y;
               const uint32_t u1 = kb < 4 ? w[r][1].x : w[r][1].y;
               const uint32_t hs0 = kb < 4 ? hs0a : hs0b, hs1 = kb < 4 ? hs1a : hs1b;
-              const uint32_t a0 = bmul2(pair_bits(u0, j, mul[j]), hs0);
-              const uint32_t a1 = bmul2(pair_bits(u1, j, mul[j]), hs1);
-              const uint32_t a2 = bmul2(pair_bits(u0, j + 1, mul[j + 1]), hs0);
-              const uint32_t a3 = bmul2(pair_bits(u1, j + 1, mul[j + 1]), hs1);
-              mma16816(acc[r], a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
-              if (kTwoTiles) mma16816(acc1[r], a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
+              const uint32_t a0 = bmul2<F16>(pair_bits(u0, j, mul[j]), hs0);
+              const uint32_t a1 = bmul2<F16>(pair_bits(u1, j, mul[j]), hs1);
+              const uint32_t a2 = bmul2<F16>(pair_bits(u0, j + 1, mul[j + 1]), hs0);
+              const uint32_t a3 = bmul2<F16>(pair_bits(u1, j + 1, mul[j + 1]), hs1);
+              mma16816<F16>(acc[r], a0, a1, a2, a3, xr[2 * kb], xr[2 * kb + 1]);
+              if (kTwoTiles) mma16816<F16>(acc1[r], a0, a1, a2, a3, yr[2 * kb], yr[2 * kb + 1]);
             }
           }
         }
@@ -755,17 +782,19 @@ cudaError_t launch_decode(DecodeBatch& b, int num_sms, cudaStream_t stream) {
   if (sched == nullptr) return cudaErrorInvalidSymbol;
   sched += 2 * (seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
   cudaError_t e;
-  if (b.m > 8) {
-    e = ensure_smem_limit<decode_kernel<true>>(kSmemLimit);
-    if (e != cudaSuccess) return e;
-    decode_kernel<true><<<static_cast<unsigned>(blocks), DecodeCfg<true>::kThreads, smem, stream>>>(
-        b, sched);
-  } else {
-    e = ensure_smem_limit<decode_kernel<false>>(kSmemLimit);
-    if (e != cudaSuccess) return e;
-    decode_kernel<false><<<static_cast<unsigned>(blocks), DecodeCfg<false>::kThreads, smem,
-                           stream>>>(b, sched);
-  }
+  auto go = [&](auto two, auto f16) -> cudaError_t {
+    constexpr bool kTwo = decltype(two)::value, kF16 = decltype(f16)::value;
+    cudaError_t err = ensure_smem_limit<decode_kernel<kTwo, kF16>>(kSmemLimit);
+    if (err != cudaSuccess) return err;
+    decode_kernel<kTwo, kF16><<<static_cast<unsigned>(blocks), DecodeCfg<kTwo>::kThreads, smem,
+                                stream>>>(b, sched);
+    return cudaSuccess;
+  };
+  if (b.m > 8)
+    e = b.in_f16 ? go(std::true_type{}, std::true_type{}) : go(std::true_type{}, std::false_type{});
+  else
+    e = b.in_f16 ? go(std::false_type{}, std::true_type{}) : go(std::false_type{}, std::false_type{});
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -202,7 +202,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16(128, kDwTileN, 1, 1);
+      const uint32_t idesc = idesc_bf16(128, kDwTileN, 1, 1, args.in_f16 != 0);
       int it = 0;
       bool ok = true;
       for (int i = 0; i < my_items && ok; ++i) {

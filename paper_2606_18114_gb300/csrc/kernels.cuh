@@ -108,6 +108,7 @@ struct TsArgs {
   int64_t m;              // tokens
   int32_t log2g;          // log2 of the group size
   int32_t out_bf16;       // 1: bf16 output
+  int32_t in_f16;         // 1: fp16 activations (else bf16)
 };
 
 // Tile of the activation operand along the token dimension.
@@ -158,6 +159,7 @@ struct DecodeBatch {
   int32_t scale_bytes;    // scale area of a slot
   int32_t stages;         // ring slots
   int32_t ubuf_bytes;     // one unit-scale buffer (two are kept)
+  int32_t in_f16;         // 1: fp16 activations in every matrix (else bf16)
 };
 
 // Reorders b.mats / b.maps (decreasing k) and sets unit0 and total_units.
@@ -170,6 +172,7 @@ struct DwArgs {
   int* status;
   int64_t m, n, k;
   int32_t accumulate;
+  int32_t in_f16;  // 1: fp16 dy and x (else bf16)
 };
 
 constexpr int kDwTileK = 128;  // lanes: input features

@@ -241,12 +241,12 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
       : "memory");
 }
 
-// Instruction descriptor, kind::f16 with bf16 A/B and fp32 D.
-// a_mn / b_mn: 0 = K-major operand, 1 = MN-major operand.
-__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n, int a_mn, int b_mn) {
+// Instruction descriptor, kind::f16 with bf16 (or, with f16, fp16) A and B — both
+// the same type — and fp32 D. a_mn / b_mn: 0 = K-major operand, 1 = MN-major operand.
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n, int a_mn, int b_mn, bool f16 = false) {
   return (1u << 4)                                   // D format: f32
-         | (1u << 7)                                 // A format: bf16
-         | (1u << 10)                                // B format: bf16
+         | (f16 ? 0u : (1u << 7))                    // A format: bf16 (1) or f16 (0)
+         | (f16 ? 0u : (1u << 10))                   // B format: the same as A
          | (static_cast<uint32_t>(a_mn) << 15)       // A major
          | (static_cast<uint32_t>(b_mn) << 16)       // B major
          | (static_cast<uint32_t>(n >> 3) << 17)     // N / 8

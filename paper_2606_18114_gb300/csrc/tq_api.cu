@@ -134,6 +134,17 @@ tq_status check_ptr(const void* p, const char* name) {
   return TQ_OK;
 }
 
+// dtype word: the output type in bits 0-7 (TQ_OUT_F32 / TQ_OUT_BF16), TQ_IN_F16
+// for fp16 activations (x, dy) instead of bf16.
+inline int out_type(int32_t dtype) { return dtype & 0xff; }
+inline bool in_f16(int32_t dtype) { return (dtype & TQ_IN_F16) != 0; }
+inline bool dtype_ok(int32_t dtype) {
+  return (dtype & ~(0xff | TQ_IN_F16)) == 0 && (out_type(dtype) == TQ_OUT_F32 || out_type(dtype) == TQ_OUT_BF16);
+}
+inline CUtensorMapDataType act_map_type(int32_t dtype) {
+  return in_f16(dtype) ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+}
+
 #define TQ_TRY(expr)                 \
   do {                               \
     const tq_status st_ = (expr);    \
@@ -159,7 +170,7 @@ tq_status fwd_checked(const void* x, int64_t m, int64_t k, const uint32_t* codes
   if (m == 0 || n == 0) return TQ_OK;
   const DeviceInfo* dev = nullptr;
   TQ_TRY(device_info(&dev));
-  const size_t ybytes = y_dtype == TQ_OUT_BF16 ? 2 : 4;
+  const size_t ybytes = out_type(y_dtype) == TQ_OUT_BF16 ? 2 : 4;
   if (k == 0) {
     cudaError_t e = cudaMemsetAsync(y, 0, static_cast<size_t>(m) * n * ybytes, stream);
     return e == cudaSuccess ? TQ_OK : cuda_fail(e, "cudaMemsetAsync");
@@ -168,8 +179,7 @@ tq_status fwd_checked(const void* x, int64_t m, int64_t k, const uint32_t* codes
   if (((n + 127) / 128) * ((m + bn - 1) / bn) >= (int64_t(1) << 31))
     return fail(TQ_ERR_UNSUPPORTED, "too many output tiles (m=%lld n=%lld)", (long long)m, (long long)n);
   CUtensorMap tb, tc;
-  TQ_TRY(make_map(&tb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, x, k, m, 64, bn,
-                  CU_TENSOR_MAP_SWIZZLE_128B));
+  TQ_TRY(make_map(&tb, act_map_type(y_dtype), 2, x, k, m, 64, bn, CU_TENSOR_MAP_SWIZZLE_128B));
   TQ_TRY(make_map(&tc, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, codes, k / 16, n, 8, 128,
                   CU_TENSOR_MAP_SWIZZLE_NONE));
   tq::TsArgs a = *proto;
@@ -181,7 +191,8 @@ tq_status fwd_checked(const void* x, int64_t m, int64_t k, const uint32_t* codes
   a.wk = k;
   a.m = m;
   a.log2g = log2_group(g);
-  a.out_bf16 = y_dtype == TQ_OUT_BF16;
+  a.out_bf16 = out_type(y_dtype) == TQ_OUT_BF16;
+  a.in_f16 = in_f16(y_dtype);
   cudaError_t e = tq::launch_ts_gemm(tq::kTsFwd, bn, tb, tc, a, dev->num_sms, stream);
   return e == cudaSuccess ? TQ_OK : cuda_fail(e, "forward launch");
 }
@@ -246,6 +257,8 @@ tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
   TQ_TRY(device_info(&dev));
   thread_local tq::DecodeBatch b;
   int used = 0;
+  // one activation type per call (checked by the callers)
+  b.in_f16 = count > 0 && in_f16(descs[0].y_dtype);
   auto flush = [&]() -> tq_status {
     if (used == 0) return TQ_OK;
     b.status = dev->status;
@@ -260,7 +273,7 @@ tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
     const tq_fwd_desc& d = descs[i];
     if (d.n == 0) continue;
     if (d.k == 0) {
-      const size_t yb = d.y_dtype == TQ_OUT_BF16 ? 2 : 4;
+      const size_t yb = out_type(d.y_dtype) == TQ_OUT_BF16 ? 2 : 4;
       cudaError_t e = cudaMemsetAsync(d.y, 0, static_cast<size_t>(m) * d.n * yb, stream);
       if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
       continue;
@@ -277,7 +290,7 @@ tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
     dm.n = d.n;
     dm.k = d.k;
     dm.log2g = log2g;
-    dm.y_bf16 = d.y_dtype == TQ_OUT_BF16;
+    dm.y_bf16 = out_type(d.y_dtype) == TQ_OUT_BF16;
     dm.unit0 = 0;
     dm.scale_mode = gpr % 4 != 0 ? tq::kDecodeScale4
                     : gpr <= 32  ? tq::kDecodeScaleUnit
@@ -291,8 +304,7 @@ tq_status check_fwd_args(const void* x, int64_t m, int64_t k, const uint32_t* co
                          const float* scales, int64_t n, int32_t g, const void* y,
                          int32_t y_dtype) {
   TQ_TRY(check_linear_shape(m, n, k, g));
-  if (y_dtype != TQ_OUT_F32 && y_dtype != TQ_OUT_BF16)
-    return fail(TQ_ERR_INVALID_ARG, "y_dtype %d", y_dtype);
+  if (!dtype_ok(y_dtype)) return fail(TQ_ERR_INVALID_ARG, "y_dtype %d", y_dtype);
   if (m == 0 || n == 0) return TQ_OK;
   TQ_TRY(check_ptr(y, "y"));
   if (k == 0) return TQ_OK;
@@ -473,6 +485,8 @@ TQ_API tq_status tq_linear_fwd_batched(const tq_fwd_desc* descs, int32_t count, 
       snprintf(msg, sizeof(msg), "descs[%d]: %s", i, g_err);
       return fail(st, "%s", msg);
     }
+    if (in_f16(d.y_dtype) != in_f16(descs[0].y_dtype))
+      return fail(TQ_ERR_INVALID_ARG, "descs[%d]: activation type differs from descs[0]", i);
   }
   return decode_checked(descs, count, m, static_cast<cudaStream_t>(stream));
 }
@@ -500,8 +514,7 @@ tq_status check_bwd_args(const void* dy, const void* x, int64_t m, int64_t n, in
   TQ_TRY(check_linear_shape(m, n, k, g));
   if (n % 8 != 0)
     return fail(TQ_ERR_UNSUPPORTED, "n=%lld: the backward kernels need n %% 8 == 0", (long long)n);
-  if (dx_dtype != TQ_OUT_F32 && dx_dtype != TQ_OUT_BF16)
-    return fail(TQ_ERR_INVALID_ARG, "dx_dtype %d", dx_dtype);
+  if (!dtype_ok(dx_dtype)) return fail(TQ_ERR_INVALID_ARG, "dx_dtype %d", dx_dtype);
   if (dx == nullptr && dw == nullptr) return fail(TQ_ERR_INVALID_ARG, "dx and dw are both NULL");
   const bool want_dx = dx != nullptr && m > 0 && k > 0;
   const bool want_dw = dw != nullptr && n > 0 && k > 0;
@@ -538,7 +551,7 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
   cudaStream_t st = static_cast<cudaStream_t>(stream);
 
   if (want_dx) {
-    const size_t dxb = dx_dtype == TQ_OUT_BF16 ? 2 : 4;
+    const size_t dxb = out_type(dx_dtype) == TQ_OUT_BF16 ? 2 : 4;
     if (n == 0) {
       cudaError_t e = cudaMemsetAsync(dx, 0, static_cast<size_t>(m) * k * dxb, st);
       if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
@@ -547,7 +560,7 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
       if (((k + 127) / 128) * ((m + bn - 1) / bn) >= (int64_t(1) << 31))
         return fail(TQ_ERR_UNSUPPORTED, "too many output tiles (m=%lld k=%lld)", (long long)m, (long long)k);
       CUtensorMap tb, tc;
-      TQ_TRY(make_map(&tb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, dy, n, m, 64, bn,
+      TQ_TRY(make_map(&tb, act_map_type(dx_dtype), 2, dy, n, m, 64, bn,
                       CU_TENSOR_MAP_SWIZZLE_128B));
       const int64_t ldt = 4 * ((n + 63) / 64);  // codes_t row length (words)
       if (codes_t != nullptr)
@@ -565,7 +578,8 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
       a.wk = k;
       a.m = m;
       a.log2g = log2_group(g);
-      a.out_bf16 = dx_dtype == TQ_OUT_BF16;
+      a.out_bf16 = out_type(dx_dtype) == TQ_OUT_BF16;
+      a.in_f16 = in_f16(dx_dtype);
       cudaError_t e = tq::launch_ts_gemm(codes_t != nullptr ? tq::kTsDxT : tq::kTsDx, bn, tb, tc,
                                          a, dev->num_sms, st);
       if (e != cudaSuccess) return cuda_fail(e, "dX launch");
@@ -582,9 +596,9 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
           (int64_t(1) << 31))
         return fail(TQ_ERR_UNSUPPORTED, "too many dW tiles (n=%lld k=%lld)", (long long)n, (long long)k);
       CUtensorMap tx, tdy;
-      TQ_TRY(make_map(&tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, x, k, m, 64, 64,
+      TQ_TRY(make_map(&tx, act_map_type(dx_dtype), 2, x, k, m, 64, 64,
                       CU_TENSOR_MAP_SWIZZLE_128B));
-      TQ_TRY(make_map(&tdy, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, dy, n, m, 64, 64,
+      TQ_TRY(make_map(&tdy, act_map_type(dx_dtype), 2, dy, n, m, 64, 64,
                       CU_TENSOR_MAP_SWIZZLE_128B));
       tq::DwArgs a{};
       a.dw = dw;
@@ -593,6 +607,7 @@ TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t
       a.n = n;
       a.k = k;
       a.accumulate = accumulate_dw != 0;
+      a.in_f16 = in_f16(dx_dtype);
       cudaError_t e = tq::launch_dw_gemm(tx, tdy, a, dev->num_sms, st);
       if (e != cudaSuccess) return cuda_fail(e, "dW launch");
     }

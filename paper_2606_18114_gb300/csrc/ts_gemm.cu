@@ -29,6 +29,7 @@
 // reduction runs over n, the scale varies along the reduction (per n), and each
 // thread picks its own 2-bit field out of the codes of 64 consecutive rows n.
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -80,27 +81,42 @@ struct TsLayout {
   static_assert(BN % 16 == 0, "epilogue chunks");
 };
 
+// Two 16-bit products in the activation type (bf16, or fp16 with F16).
+template <bool F16>
 __device__ __forceinline__ uint32_t bmul2(uint32_t a, uint32_t b) {
   uint32_t d;
-  asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  if constexpr (F16)
+    asm("mul.rn.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+  else
+    asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
   return d;
 }
 
-__device__ __forceinline__ uint32_t half_scale_pair(float lo, float hi) {
-  // bf16(s)/2 in both halves; s/2 is exact in fp32 and rounding commutes with it.
-  const __nv_bfloat16 l = __float2bfloat16_rn(0.5f * lo);
-  const __nv_bfloat16 h = __float2bfloat16_rn(0.5f * hi);
-  return static_cast<uint32_t>(__bfloat16_as_ushort(l)) |
-         (static_cast<uint32_t>(__bfloat16_as_ushort(h)) << 16);
+// s / 2 rounded to the activation type, as its 16 bits.
+template <bool F16>
+__device__ __forceinline__ uint16_t half_scale_bits(float s) {
+  if constexpr (F16)
+    return __half_as_ushort(__float2half_rn(0.5f * s));
+  else
+    return __bfloat16_as_ushort(__float2bfloat16_rn(0.5f * s));
 }
 
-// 16 codes of one word -> 8 bf16x2 A-operand columns, times the scale pair.
+template <bool F16>
+__device__ __forceinline__ uint32_t half_scale_pair(float lo, float hi) {
+  // round(s)/2 in both halves; s/2 is exact in fp32 and rounding commutes with it.
+  return static_cast<uint32_t>(half_scale_bits<F16>(lo)) |
+         (static_cast<uint32_t>(half_scale_bits<F16>(hi)) << 16);
+}
+
+// 16 codes of one word -> 8 A-operand columns of two 16-bit values, times the
+// scale pair (the codes expand to +-2 = 0x4000 / 0xC000 in bf16 and fp16 alike).
+template <bool F16>
 __device__ __forceinline__ void expand_word(uint32_t w, uint32_t hs, uint32_t* a) {
 #pragma unroll
-  for (int j = 0; j < 8; ++j) a[j] = bmul2((w << (14 - 2 * j)) & 0xC000C000u, hs);
+  for (int j = 0; j < 8; ++j) a[j] = bmul2<F16>((w << (14 - 2 * j)) & 0xC000C000u, hs);
 }
 
-template <int MODE, int BN>
+template <int MODE, int BN, bool F16>
 __global__ void __launch_bounds__(kThreads, 1)
     ts_gemm_kernel(const __grid_constant__ CUtensorMap tmap_b,
                    const __grid_constant__ CUtensorMap tmap_codes, const TsArgs args) {
@@ -199,7 +215,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16(128, BN, 0, 0);
+      constexpr uint32_t idesc = idesc_bf16(128, BN, 0, 0, F16);
       int it = 0;
       bool ok = true;
       for (int i = 0; i < my_tiles && ok; ++i) {
@@ -348,13 +364,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!lanes_wait(full_bar(s), (it / kSmem) & 1, status)) break;
         const uint4 cw = *reinterpret_cast<const uint4*>(smem + s * L::kStageBytes + L::kBBytes +
                                                          r_local * 32 + wg * 16);
-        const uint32_t hs_lo = half_scale_pair(sc.x, sc.x);
-        const uint32_t hs_hi = half_scale_pair(sc.y, sc.y);
+        const uint32_t hs_lo = half_scale_pair<F16>(sc.x, sc.x);
+        const uint32_t hs_hi = half_scale_pair<F16>(sc.y, sc.y);
         uint32_t a[32];
-        expand_word(cw.x, hs_lo, a + 0);
-        expand_word(cw.y, hs_lo, a + 8);
-        expand_word(cw.z, hs_hi, a + 16);
-        expand_word(cw.w, hs_hi, a + 24);
+        expand_word<F16>(cw.x, hs_lo, a + 0);
+        expand_word<F16>(cw.y, hs_lo, a + 8);
+        expand_word<F16>(cw.z, hs_hi, a + 16);
+        expand_word<F16>(cw.w, hs_hi, a + 24);
         if (!a_free(it)) break;
         publish(as, a);
       }
@@ -374,8 +390,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (n_b < args.wn) r.y = __ldg(args.scales + n_b * gpr + gk);
         return r;
       };
-      __nv_bfloat16* sbuf =
-          reinterpret_cast<__nv_bfloat16*>(smem + L::kScaleOff) + (wg * 4 + quad) * 128;
+      uint16_t* sbuf = reinterpret_cast<uint16_t*>(smem + L::kScaleOff) + (wg * 4 + quad) * 128;
       float2 p0 = load_sc(cur), p1 = load_sc(cursor_at(1));
       if (MODE == kTsDxT) {
         // codes_t: this thread's row k of the transposed codes holds rows n along it,
@@ -386,9 +401,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float2 sc = p0;
           p0 = p1;
           p1 = load_sc(pre);
-          __nv_bfloat16* sb = sbuf + (it & 1) * 64;
-          sb[lane] = __float2bfloat16_rn(0.5f * sc.x);
-          sb[lane + 32] = __float2bfloat16_rn(0.5f * sc.y);
+          uint16_t* sb = sbuf + (it & 1) * 64;
+          sb[lane] = half_scale_bits<F16>(sc.x);
+          sb[lane + 32] = half_scale_bits<F16>(sc.y);
           __syncwarp();
           if (!lanes_wait(full_bar(s), (it / kSmem) & 1, status)) break;
           const uint4 cw = *reinterpret_cast<const uint4*>(smem + s * L::kStageBytes + L::kBBytes +
@@ -402,7 +417,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t pr[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
 #pragma unroll
             for (int j = 0; j < 8; ++j)
-              a[8 * q + j] = bmul2((words[q] << (14 - 2 * j)) & 0xC000C000u, pr[j]);
+              a[8 * q + j] = bmul2<F16>((words[q] << (14 - 2 * j)) & 0xC000C000u, pr[j]);
           }
           if (!a_free(it)) break;
           publish(as, a);
@@ -420,9 +435,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float2 sc = p0;
         p0 = p1;
         p1 = load_sc(pre);
-        __nv_bfloat16* sb = sbuf + (it & 1) * 64;
-        sb[lane] = __float2bfloat16_rn(0.5f * sc.x);
-        sb[lane + 32] = __float2bfloat16_rn(0.5f * sc.y);
+        uint16_t* sb = sbuf + (it & 1) * 64;
+        sb[lane] = half_scale_bits<F16>(sc.x);
+        sb[lane + 32] = half_scale_bits<F16>(sc.y);
         __syncwarp();
         if (!lanes_wait(full_bar(s), (it / kSmem) & 1, status)) break;
         const uint32_t* tile =
@@ -434,7 +449,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t w0 = tile[(2 * p) * 8 + xw];
           const uint32_t w1 = tile[(2 * p + 1) * 8 + xw];
           const uint32_t t = (__byte_perm(w0, w1, sel) << shift) & 0xC000C000u;
-          a[p] = bmul2(t, spair[p]);
+          a[p] = bmul2<F16>(t, spair[p]);
         }
         if (!a_free(it)) break;
         publish(as, a);
@@ -452,7 +467,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int MODE, int BN>
+template <int MODE, int BN, bool F16>
 cudaError_t launch_impl(const CUtensorMap& tb, const CUtensorMap& tc, const TsArgs& a,
                         int num_sms, cudaStream_t stream) {
   using L = TsLayout<MODE, BN>;
@@ -460,8 +475,8 @@ cudaError_t launch_impl(const CUtensorMap& tb, const CUtensorMap& tc, const TsAr
   // tensor-memory columns).
   size_t smem = L::kBytes + 1024;
   if (smem < 116 * 1024) smem = 116 * 1024;
-  auto kern = ts_gemm_kernel<MODE, BN>;
-  cudaError_t e = ensure_smem_limit<ts_gemm_kernel<MODE, BN>>(static_cast<int>(smem));
+  auto kern = ts_gemm_kernel<MODE, BN, F16>;
+  cudaError_t e = ensure_smem_limit<ts_gemm_kernel<MODE, BN, F16>>(static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   const int64_t rows = MODE == kTsFwd ? a.wn : a.wk;
   const int64_t tiles = ((rows + 127) / 128) * ((a.m + BN - 1) / BN);
@@ -474,18 +489,27 @@ cudaError_t launch_impl(const CUtensorMap& tb, const CUtensorMap& tc, const TsAr
 
 int ts_tile_tokens(int mode, int64_t m) { return m <= 16 ? 16 : 256; }
 
-cudaError_t launch_ts_gemm(int mode, int bn, const CUtensorMap& tb, const CUtensorMap& tc,
-                           const TsArgs& a, int num_sms, cudaStream_t stream) {
+namespace {
+template <bool F16>
+cudaError_t launch_typed(int mode, int bn, const CUtensorMap& tb, const CUtensorMap& tc,
+                         const TsArgs& a, int num_sms, cudaStream_t stream) {
   if (mode == kTsFwd) {
-    if (bn == 256) return launch_impl<kTsFwd, 256>(tb, tc, a, num_sms, stream);
+    if (bn == 256) return launch_impl<kTsFwd, 256, F16>(tb, tc, a, num_sms, stream);
   } else if (mode == kTsDx) {
-    if (bn == 16) return launch_impl<kTsDx, 16>(tb, tc, a, num_sms, stream);
-    if (bn == 256) return launch_impl<kTsDx, 256>(tb, tc, a, num_sms, stream);
+    if (bn == 16) return launch_impl<kTsDx, 16, F16>(tb, tc, a, num_sms, stream);
+    if (bn == 256) return launch_impl<kTsDx, 256, F16>(tb, tc, a, num_sms, stream);
   } else if (mode == kTsDxT) {
-    if (bn == 16) return launch_impl<kTsDxT, 16>(tb, tc, a, num_sms, stream);
-    if (bn == 256) return launch_impl<kTsDxT, 256>(tb, tc, a, num_sms, stream);
+    if (bn == 16) return launch_impl<kTsDxT, 16, F16>(tb, tc, a, num_sms, stream);
+    if (bn == 256) return launch_impl<kTsDxT, 256, F16>(tb, tc, a, num_sms, stream);
   }
   return cudaErrorInvalidValue;
+}
+}  // namespace
+
+cudaError_t launch_ts_gemm(int mode, int bn, const CUtensorMap& tb, const CUtensorMap& tc,
+                           const TsArgs& a, int num_sms, cudaStream_t stream) {
+  return a.in_f16 ? launch_typed<true>(mode, bn, tb, tc, a, num_sms, stream)
+                  : launch_typed<false>(mode, bn, tb, tc, a, num_sms, stream);
 }
 
 }  // namespace tq

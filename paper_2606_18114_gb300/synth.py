@@ -26,6 +26,7 @@ __all__ = [
     "rng",
     "latent_weights",
     "activations_bf16",
+    "activations_f16",
     "MAMBA2_1P3B",
 ]
 
@@ -58,6 +59,15 @@ def latent_weights(n: int, k: int, seed: int, dist: str = "gauss", std: float = 
     else:
         raise ValueError(f"unknown weight distribution {dist!r}")
     return np.ascontiguousarray(w)
+
+
+def activations_f16(m: int, k: int, seed: int, std: float = 1.0, stream: str = "x") -> torch.Tensor:
+    """fp16 CPU tensor ``[m, k]``: the draw of :func:`activations_bf16`, rounded to fp16."""
+    g = rng(seed, stream)
+    a = g.standard_normal((m, k), dtype=np.float32)
+    if std != 1.0:
+        a *= np.float32(std)
+    return torch.from_numpy(a).to(torch.float16).contiguous()
 
 
 def activations_bf16(m: int, k: int, seed: int, std: float = 1.0, stream: str = "x") -> torch.Tensor:

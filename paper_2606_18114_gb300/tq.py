@@ -37,6 +37,7 @@ __all__ = [
 
 OUT_F32 = 0
 OUT_BF16 = 1
+IN_F16 = 0x100  # flag: fp16 activations (x, dy) instead of bf16
 STATUS = {0: "TQ_OK", 1: "TQ_ERR_INVALID_ARG", 2: "TQ_ERR_UNSUPPORTED", 3: "TQ_ERR_CUDA",
           4: "TQ_ERR_TIMEOUT"}
 # Every symbol include/tq.h declares.
@@ -251,15 +252,25 @@ def _out_code(dtype) -> int:
     raise ValueError(f"unsupported output dtype {dtype}")
 
 
+def _in_flag(act: Optional[torch.Tensor]) -> int:
+    """IN_F16 for fp16 activations, 0 for bf16 (the activation type rides on the
+    output-type word of the C calls)."""
+    if act is None or act.dtype == torch.bfloat16:
+        return 0
+    if act.dtype == torch.float16:
+        return IN_F16
+    raise ValueError(f"unsupported activation dtype {act.dtype}")
+
+
 def linear_fwd(x: torch.Tensor, codes: torch.Tensor, scales: torch.Tensor, g: int,
                out_dtype=torch.float32, y: Optional[torch.Tensor] = None, stream=None):
-    """W1.58A16 forward ``y = x W^T`` for bf16 ``x [M, K]``; returns ``y [M, N]``."""
+    """W1.58A16 forward ``y = x W^T`` for bf16 (or fp16) ``x [M, K]``; returns ``y [M, N]``."""
     m, k = x.shape
     n = codes.shape[0]
     if y is None:
         y = torch.empty((m, n), dtype=out_dtype, device=x.device)
     _check(load().tq_linear_fwd(_ptr(x), m, k, _ptr(codes), _ptr(scales), n, g, _ptr(y),
-                                _out_code(y.dtype), _stream(stream)))
+                                _out_code(y.dtype) | _in_flag(x), _stream(stream)))
     return y
 
 
@@ -291,7 +302,8 @@ def linear_bwd(dy: torch.Tensor, x: Optional[torch.Tensor], codes: torch.Tensor,
         dw = None
     _check(load().tq_linear_bwd(_ptr(dy), _ptr(x), m, n, k, _ptr(codes), _ptr(codes_t),
                                 _ptr(scales), g,
-                                _ptr(dx), _out_code(dx.dtype) if dx is not None else OUT_F32,
+                                _ptr(dx), (_out_code(dx.dtype) if dx is not None else OUT_F32)
+                                | _in_flag(dy),
                                 _ptr(dw), int(accumulate_dw), _stream(stream)))
     return dx, dw
 
@@ -313,7 +325,8 @@ def linear_bwd_noalloc(dy: torch.Tensor, x: Optional[torch.Tensor], codes: torch
     if not want_dw:
         dw = None
     _check(load().tq_linear_bwd_noalloc(_ptr(dy), _ptr(x), m, n, k, _ptr(codes), _ptr(scales), g,
-                                        _ptr(dx), _out_code(dx.dtype) if dx is not None else OUT_F32,
+                                        _ptr(dx), (_out_code(dx.dtype) if dx is not None else OUT_F32)
+                                        | _in_flag(dy),
                                         _ptr(dw), int(accumulate_dw), _stream(stream)))
     return dx, dw
 
@@ -328,7 +341,8 @@ def fwd_batch(items: Sequence[dict]):
     for i, it in enumerate(items):
         codes = it["codes"]
         arr[i] = FwdDesc(_ptr(it["x"]), _ptr(codes), _ptr(it["scales"]), _ptr(it["y"]),
-                         codes.shape[0], codes.shape[1] * 16, it["g"], _out_code(it["y"].dtype))
+                         codes.shape[0], codes.shape[1] * 16, it["g"],
+                         _out_code(it["y"].dtype) | _in_flag(it["x"]))
     return arr
 
 

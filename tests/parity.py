@@ -74,3 +74,15 @@ def check_close(got, ref: np.ndarray, what: str, rel_frob=REL_FROB, max_rel_rms=
     assert relf <= rel_frob, f"{what}: relative Frobenius error {relf:.3e} > {rel_frob}"
     assert mx <= max_rel_rms * rms, f"{what}: max error {mx:.3e} > {max_rel_rms} * rms {rms:.3e}"
     return relf, mx / rms if rms > 0 else 0.0
+
+
+def validated_w_hat(w: np.ndarray, g: int, codes_gpu, scales_gpu, zeros_gpu) -> np.ndarray:
+    """The dequantized weights the GPU products use, for comparing those products:
+    the GPU codes are first checked against the oracle (identical outside
+    near-ties, where either rounding is correct), then expanded with the oracle's
+    fp64-exact scales. Building W^ from the oracle's own codes instead would charge
+    a product with s * x for every near-tie weight the two sides round apart."""
+    n, k = w.shape
+    ref = O.quantize(w, g)
+    check_quantize(w, g, codes_gpu, scales_gpu, zeros_gpu, ref=ref)
+    return O.dequantize(codes_u32(codes_gpu), ref[1], k, g)

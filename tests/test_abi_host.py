@@ -187,3 +187,19 @@ def test_decoupled_and_alpha_grad_reject_before_launch(lib):
     assert ag(FAKE, FAKE, 8, 256, 128, None, None) == 1                   # null dalpha
     assert ag(FAKE, FAKE, -1, 256, 128, FAKE, None) == 1                  # negative size
     assert ag(FAKE, FAKE, 0, 256, 128, FAKE, None) == 0                   # empty
+
+
+def test_activation_flag_checked(lib):
+    """The output-type word takes TQ_IN_F16 and nothing else beyond the output type;
+    a batched decode takes one activation type."""
+    from paper_2606_18114_gb300.tq import FwdDesc
+    f = lib.tq_linear_fwd
+    assert f(FAKE, 4, 256, FAKE, FAKE, 64, 128, FAKE, 0x200, None) == 1   # unknown flag
+    assert f(FAKE, 4, 256, FAKE, FAKE, 64, 128, FAKE, 0x102, None) == 1   # bad output type
+    b = lib.tq_linear_bwd
+    assert b(FAKE, FAKE, 4, 64, 256, FAKE, None, FAKE, 128, FAKE, 0x400, None, 0, None) == 1
+    arr = (FwdDesc * 2)()
+    arr[0] = FwdDesc(FAKE, FAKE, FAKE, FAKE, 64, 256, 128, 0)
+    arr[1] = FwdDesc(FAKE, FAKE, FAKE, FAKE, 64, 256, 128, 0x100)
+    assert lib.tq_linear_fwd_batched(arr, 2, 4, None) == 1
+    assert b"activation type" in lib.tq_last_error()

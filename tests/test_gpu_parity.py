@@ -9,7 +9,7 @@ import torch
 
 from oracle import tq_oracle as O
 from paper_2606_18114_gb300 import synth
-from parity import check_close, check_quantize, codes_u32, to_np
+from parity import check_close, check_quantize, codes_u32, to_np, validated_w_hat
 
 pytestmark = pytest.mark.gpu
 
@@ -165,10 +165,8 @@ def _setup(tq, n, k, m, g, seed=0, dy_std=1.0, dist="gauss"):
     w = synth.latent_weights(n, k, seed=seed, dist=dist)
     x = synth.activations_bf16(m, k, seed=seed, stream="x")
     dy = synth.activations_bf16(m, n, seed=seed, std=dy_std, stream="dy")
-    ref = O.quantize(w, g)
-    w_hat = O.dequantize(ref[0], ref[1], k, g)
     codes, s, z = _quant(tq, w, g)
-    return w, x, dy, w_hat, codes, s
+    return w, x, dy, validated_w_hat(w, g, codes, s, z), codes, s
 
 
 @pytest.mark.parametrize("n,k,m,g", [
@@ -297,11 +295,10 @@ def test_batched_decode_mixed(tq):
     for i, (n, k, g, dt) in enumerate(specs):
         w = synth.latent_weights(n, k, seed=200 + i)
         x = synth.activations_bf16(11, k, seed=200 + i)
-        codes, s, _ = _quant(tq, w, g)
-        ref = O.quantize(w, g)
+        codes, s, z = _quant(tq, w, g)
         items.append(dict(x=x.cuda(), codes=codes, scales=s, g=g,
                           y=torch.empty((11, n), device="cuda", dtype=dt),
-                          ref=O.linear_fwd(x, O.dequantize(ref[0], ref[1], k, g))))
+                          ref=O.linear_fwd(x, validated_w_hat(w, g, codes, s, z))))
     tq.linear_fwd_batched(items, 11)
     tq.device_status()
     for i, it in enumerate(items):
@@ -314,9 +311,8 @@ def test_batched_decode_matches_single(tq):
     for i, (n, k) in enumerate([(520, 256), (256, 512), (520, 256), (136, 1024)]):
         w = synth.latent_weights(n, k, seed=100 + i)
         x = synth.activations_bf16(4, k, seed=100 + i)
-        codes, s, _ = _quant(tq, w, 128)
-        ref = O.quantize(w, 128)
-        w_hat = O.dequantize(ref[0], ref[1], k, 128)
+        codes, s, z = _quant(tq, w, 128)
+        w_hat = validated_w_hat(w, 128, codes, s, z)
         mats.append(dict(x=x.cuda(), codes=codes, scales=s, g=128,
                          y=torch.empty((4, n), device="cuda"), ref=O.linear_fwd(x, w_hat)))
     tq.linear_fwd_batched(mats, 4)
@@ -384,7 +380,7 @@ def test_prefill_sweep_all_group_sizes(tq, proj, g, dist):
     codes, s, z = _quant(tq, w, g)
     flips, ties = check_quantize(w, g, codes, s, z, ref=ref)
     assert flips <= ties
-    w_hat = O.dequantize(ref[0], ref[1], k, g)
+    w_hat = O.dequantize(codes_u32(codes), ref[1], k, g)  # the GPU codes, checked above
     y = tq.linear_fwd(xd, codes, s, g)
     ct = tq.codes_transpose(codes, k)
     dx, dw = tq.linear_bwd(dyd, xd, codes, s, k, g, codes_t=ct)
@@ -397,3 +393,40 @@ def test_prefill_sweep_all_group_sizes(tq, proj, g, dist):
     check_close(to_np(dx[sel]), O.linear_bwd_dx(dy, w_hat, rows), f"dX rows {proj} g={g} {dist}")
     check_close(to_np(dw[torch.from_numpy(nrows).cuda()]), O.linear_bwd_dw(dy, x, nrows),
                 f"dW rows {proj} g={g} {dist}")
+
+
+# ------------------------------------------------------------------ extreme shapes
+@pytest.mark.parametrize("m", [1, 5, 12])
+def test_decode_long_reduction(tq, m):
+    """Decode over a 16384-long reduction: 32 segments per 256-row unit, a ragged
+    last unit of 44 rows."""
+    n, k, g = 300, 16384, 128
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=51)
+    y = tq.linear_fwd(x.cuda(), codes, s, g)
+    tq.device_status()
+    check_close(to_np(y), O.linear_fwd(x, w_hat), f"Y m={m} k={k}")
+
+
+def test_prefill_few_rows_many_tokens(tq):
+    """64 weight rows (half a tile) against 40000 tokens (157 token tiles with a
+    ragged last one), all three products."""
+    n, k, m, g = 64, 512, 40000, 64
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=52, dy_std=1e-2)
+    xd, dyd = x.cuda(), dy.cuda()
+    y = tq.linear_fwd(xd, codes, s, g)
+    dx, dw = tq.linear_bwd(dyd, xd, codes, s, k, g, codes_t=tq.codes_transpose(codes, k))
+    tq.device_status()
+    rows = np.sort(np.random.default_rng(52).choice(m, 256, replace=False))
+    sel = torch.from_numpy(rows).cuda()
+    check_close(to_np(y[sel]), O.linear_fwd(x, w_hat, rows), "Y rows")
+    check_close(to_np(dx[sel]), O.linear_bwd_dx(dy, w_hat, rows), "dX rows")
+    check_close(to_np(dw), O.linear_bwd_dw(dy, x), "dW (40000-token reduction)")
+
+
+def test_dw_long_token_reduction(tq):
+    """dW over 131072 tokens (2048 k-blocks per tile, fewer tiles than SMs)."""
+    n, k, m, g = 256, 384, 131072, 128
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=53, dy_std=1e-2)
+    _, dw = tq.linear_bwd(dy.cuda(), x.cuda(), codes, s, k, g, want_dx=False)
+    tq.device_status()
+    check_close(to_np(dw), O.linear_bwd_dw(dy, x), "dW (131072 tokens)")

@@ -7,7 +7,7 @@ import torch
 
 from oracle import tq_oracle as O
 from paper_2606_18114_gb300 import synth
-from parity import check_close
+from parity import check_close, validated_w_hat
 
 FAKE = 1 << 20
 
@@ -44,15 +44,14 @@ def test_noalloc_matches_explicit_codes_t(tq, n, k, m):
     w = torch.from_numpy(synth.latent_weights(n, k, seed=n)).cuda()
     x = synth.activations_bf16(m, k, seed=n, stream="x").cuda()
     dy = synth.activations_bf16(m, n, seed=n, std=1e-2, stream="dy").cuda()
-    codes, s, _ = tq.quantize(w, g)
+    codes, s, z = tq.quantize(w, g)
     codes_t = tq.codes_transpose(codes, k)
     dx1, dw1 = tq.linear_bwd(dy, x, codes, s, k, g, codes_t=codes_t)
     dx2, dw2 = tq.linear_bwd_noalloc(dy, x, codes, s, k, g)
     tq.device_status()
     assert torch.equal(dx1, dx2) and torch.equal(dw1, dw2)
     # and the oracle, on the dequantised weights
-    ref_codes, ref_s, _, _ = O.quantize(w.cpu().numpy(), g)
-    w_hat = O.dequantize(ref_codes, ref_s, k, g)
+    w_hat = validated_w_hat(w.cpu().numpy(), g, codes, s, z)
     check_close(dx2, O.linear_bwd_dx(dy.float().cpu(), w_hat), "dX (no-alloc)")
 
 
