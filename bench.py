@@ -171,13 +171,13 @@ def whole_job(units_per_rank: float, world: int, max_ms: float, steps: int):
 class Prefill:
     """Device-resident inputs/outputs of one projection's prefill step."""
 
-    def __init__(self, tq, n, k, m, g, seed):
+    def __init__(self, tq, n, k, m, g, seed, act=torch.bfloat16):
         gen = torch.Generator(device="cuda")
         gen.manual_seed(seed)
         self.tq, self.n, self.k, self.m, self.g = tq, n, k, m, g
         self.w = torch.randn((n, k), generator=gen, device="cuda") * 0.02
-        self.x = torch.randn((m, k), generator=gen, device="cuda").to(torch.bfloat16)
-        self.dy = (torch.randn((m, n), generator=gen, device="cuda") * 1e-2).to(torch.bfloat16)
+        self.x = torch.randn((m, k), generator=gen, device="cuda").to(act)
+        self.dy = (torch.randn((m, n), generator=gen, device="cuda") * 1e-2).to(act)
         self.codes = torch.empty((n, k // 16), dtype=torch.int32, device="cuda")
         self.codes_t = torch.empty((k, 4 * ((n + 63) // 64)), dtype=torch.int32, device="cuda")
         self.s = torch.empty((n, k // g), dtype=torch.float32, device="cuda")
@@ -373,9 +373,10 @@ def quantize_sweep(tq, steps, warmup):
     return {"ms": round(ms, 3), "GB/s": round(nbytes / ms / 1e6, 1), "bytes": nbytes}
 
 
-def out_proj_step(tq, steps, warmup):
-    """The same step on the out_proj shape (W [2048, 4096], X [16384, 4096])."""
-    p = Prefill(tq, OUT_PROJ[0], OUT_PROJ[1], M_PREFILL, G, seed=8)
+def out_proj_step(tq, steps, warmup, shape=OUT_PROJ, act=torch.bfloat16):
+    """The same step on another shape (default out_proj: W [2048, 4096], X [16384, 4096])
+    or activation type."""
+    p = Prefill(tq, shape[0], shape[1], M_PREFILL, G, seed=8, act=act)
     total_ms, per = time_prefill(p, steps, warmup, 1)
     ms = total_ms / steps
     gemm = 2.0 * p.m * p.n * p.k
@@ -793,6 +794,7 @@ def main():
             "decode_48_layers": decode_sweep(tq, (1, 4, 16), 20, 3),
             "quantize_48_layers_g128": quantize_sweep(tq, 5, 2),
             "out_proj_step": out_proj_step(tq, 200, 10),
+            "in_proj_step_fp16_activations": out_proj_step(tq, 200, 10, IN_PROJ, torch.float16),
             "sweep_48_layers": g_sweep(tq),
             "adamw_requantize_g128": adamw_sweep(tq, 5, 2),
             "decoupled_in_proj": decoupled_sweep(tq, 20, 3),
