@@ -257,39 +257,58 @@ cudaError_t launch_g(const QuantBatch<kMax>& b, int g, int* status, int num_sms,
   }
 }
 
-// codes [n][k/16] -> codes_t [k][ldt]: a 128 x 128 (n x k) tile per block. The tile's
-// 128 rows x 8 code words are read with one 32-byte sector per row, and each
-// output row k receives 8 consecutive words (one sector) of the transposed tile.
-__device__ __forceinline__ int code_pos(int i) { return 16 * (i & 1) + 2 * (i >> 1); }
+// codes [n][k/16] -> codes_t [k][ldt]. Each thread owns one 16 x 16 block of 2-bit
+// codes (16 rows n of one code word c) and transposes it in registers with four
+// levels of block swaps (8, 4, 2, 1 fields; the two byte-sized levels are byte
+// permutes). Field p of a word holds element i(p) = 2 (p % 8) + p / 8 (the packing
+// puts the even elements in the low half), so the rows are loaded in the order
+// i(q) and the transposed word p is stored as output row i(p): the plain
+// transpose then lands every element at its packed position. A warp covers 8
+// consecutive words x 4 consecutive 16-row groups (32-byte reads, 16-byte writes);
+// rows past n read as 0, which writes the zero padding of the last words.
+__device__ __forceinline__ void swap_fields(uint32_t& a, uint32_t& c, int shift, uint32_t mask) {
+  const uint32_t t = ((a >> shift) ^ c) & mask;
+  c ^= t;
+  a ^= t << shift;
+}
 
 __global__ void __launch_bounds__(256) transpose_codes_kernel(const uint32_t* __restrict__ codes,
                                                               int64_t n, int64_t k,
                                                               uint32_t* __restrict__ codes_t,
                                                               int64_t ldt) {
-  __shared__ uint32_t tile[128][9];
-  const int64_t n0 = static_cast<int64_t>(blockIdx.y) * 128;
-  const int64_t k0 = static_cast<int64_t>(blockIdx.x) * 128;
+  const int tid = threadIdx.x;
+  const int64_t c = static_cast<int64_t>(blockIdx.x) * 32 + (tid & 7) + 8 * ((tid >> 5) & 3);
+  const int64_t r16 = static_cast<int64_t>(blockIdx.y) * 8 + ((tid >> 3) & 3) + 4 * (tid >> 7);
   const int64_t words = k >> 4;
+  if (c >= words || r16 >= ldt) return;
+  uint32_t t[16];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int idx = threadIdx.x + 256 * i;
-    const int r = idx >> 3, c = idx & 7;
-    const int64_t row = n0 + r, col = (k0 >> 4) + c;
-    tile[r][c] = (row < n && col < words) ? codes[row * words + col] : 0u;
+  for (int q = 0; q < 16; ++q) {
+    const int64_t row = 16 * r16 + 2 * (q & 7) + (q >> 3);
+    t[q] = row < n ? __ldg(codes + row * words + c) : 0u;
   }
-  __syncthreads();
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int idx = threadIdx.x + 256 * i;
-    const int kk = idx >> 3, ww = idx & 7;
-    const int64_t kg = k0 + kk, wg = (n0 >> 4) + ww;
-    if (kg >= k || wg >= ldt) continue;
-    const int c = kk >> 4, sh = code_pos(kk & 15);
-    uint32_t out = 0;
-#pragma unroll
-    for (int j = 0; j < 16; ++j) out |= ((tile[16 * ww + j][c] >> sh) & 3u) << code_pos(j);
-    codes_t[kg * ldt + wg] = out;
+  for (int w = 0; w < 8; ++w) {
+    const uint32_t a = t[w], b = t[w + 8];
+    t[w] = __byte_perm(a, b, 0x5410);
+    t[w + 8] = __byte_perm(a, b, 0x7632);
   }
+#pragma unroll
+  for (int w = 0; w < 16; ++w) {
+    if (w & 4) continue;
+    const uint32_t a = t[w], b = t[w + 4];
+    t[w] = __byte_perm(a, b, 0x6240);
+    t[w + 4] = __byte_perm(a, b, 0x7351);
+  }
+#pragma unroll
+  for (int w = 0; w < 16; ++w)
+    if (!(w & 2)) swap_fields(t[w], t[w + 2], 4, 0x0F0F0F0Fu);
+#pragma unroll
+  for (int w = 0; w < 16; ++w)
+    if (!(w & 1)) swap_fields(t[w], t[w + 1], 2, 0x33333333u);
+  uint32_t* out = codes_t + 16 * c * ldt + r16;
+#pragma unroll
+  for (int p = 0; p < 16; ++p) out[(2 * (p & 7) + (p >> 3)) * ldt] = t[p];
 }
 
 }  // namespace
@@ -365,7 +384,7 @@ cudaError_t launch_alpha_grad(const float* dw, const uint32_t* codes, int64_t n,
 cudaError_t launch_transpose_codes(const uint32_t* codes, int64_t n, int64_t k, uint32_t* codes_t,
                                    cudaStream_t stream) {
   const int64_t ldt = 4 * ((n + 63) / 64);
-  dim3 grid(static_cast<unsigned>((k + 127) / 128), static_cast<unsigned>((n + 127) / 128));
+  dim3 grid(static_cast<unsigned>((k / 16 + 31) / 32), static_cast<unsigned>((ldt + 7) / 8));
   transpose_codes_kernel<<<grid, 256, 0, stream>>>(codes, n, k, codes_t, ldt);
   return cudaGetLastError();
 }

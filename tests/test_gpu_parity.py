@@ -194,13 +194,16 @@ def test_linear_parity(tq, n, k, m, g):
     check_close(dw, O.linear_bwd_dw(dy, x), "dW")
 
 
-@pytest.mark.parametrize("n,k", [(200, 192), (64, 64), (520, 1024), (1000, 2048), (8512, 2048)])
+@pytest.mark.parametrize("n,k", [(200, 192), (64, 64), (17, 16), (130, 528), (520, 1024),
+                                 (1000, 2048), (2048, 4096), (8512, 2048)])
 def test_codes_transpose_layout(tq, n, k):
-    """tq_codes_transpose against the oracle's packing of the transposed codes."""
+    """tq_codes_transpose against the oracle's packing of the transposed codes; the
+    output starts as all ones, so the zero padding past n is written, not assumed."""
     rs = np.random.default_rng(n + k)
     c = rs.choice(np.array([-1, 0, 1], dtype=np.int8), size=(n, k))
     codes = torch.from_numpy(O.pack(c).view(np.int32)).cuda()
-    ct = tq.codes_transpose(codes, k)
+    ct = torch.full((k, 4 * ((n + 63) // 64)), -1, dtype=torch.int32, device="cuda")
+    tq.codes_transpose(codes, k, out=ct)
     tq.device_status()
     npad = 64 * ((n + 63) // 64)
     cpad = np.zeros((k, npad), dtype=np.int8)
