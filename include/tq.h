@@ -143,6 +143,43 @@ TQ_API tq_status tq_quantize_decoupled(const float* w, int64_t n, int64_t k, int
 TQ_API tq_status tq_alpha_grad(const float* dw, const uint32_t* codes, int64_t n, int64_t k,
                                int32_t g, float* dalpha, void* stream);
 
+/*
+ * tq_quantize_with_scales — the quantizer of the learnable-scale variant (§4,
+ * "Zero-Ratio Collapse": s_g trained as a parameter instead of recomputed as the
+ * absmean): the codes are decided against the caller's scales,
+ *   c = round(clip(w / s_g, -1, 1))   (the fp32 quotient, rounding half to even),
+ * for a scale of either sign (for s_g < 0 the codes flip with it, so s_g * c still
+ * approximates w; s_g = 0 gives the sign of w, and 0 for w = 0).
+ *   scales   fp32 [n][k/g]: the current s_g (device, 16-byte aligned); read only.
+ *   codes, zero_counts   out: as tq_quantize.
+ *   Other arguments, layouts and errors as tq_quantize; the forward and backward
+ *   products take these scales as they take the absmean.
+ */
+TQ_API tq_status tq_quantize_with_scales(const float* w, int64_t n, int64_t k, int32_t g,
+                                         const float* scales, uint32_t* codes,
+                                         int32_t* zero_counts, void* stream);
+
+/*
+ * tq_scale_grad — gradient of the learnable scale. The paper does not give it;
+ * this library takes the chain rule through W^ = s * round(clip(w / s)) with the
+ * rounding passed straight through (the rule §3.1 applies to the latent weights):
+ *   dW^/ds = c - q [|q| < 1],  q = w / s, so
+ *   dscales[n][j] = sum_i dW^_i c_i - (1/s) sum_{i : |w_i| < |s|} dW^_i w_i
+ * over group j of row n, where dW^ is the dW of tq_linear_bwd. The test |w| < |s|
+ * compares the fp32 inputs exactly; for s = 0 the second sum is empty.
+ *   w        fp32 [n][k], the latent weights the codes came from (device, 16-byte aligned).
+ *   dw       fp32 [n][k] (device, 16-byte aligned).
+ *   codes    uint32 [n][k/16] of tq_quantize_with_scales for (w, scales).
+ *   scales   fp32 [n][k/g] (device, 4-byte aligned).
+ *   dscales  out: fp32 [n][k/g] (device, 4-byte aligned).
+ *   Summation: each 16-weight word in weight order, then the group's words as a
+ *   binary tree, both sums in fp32, then one fp32 division. Requires k % g == 0;
+ *   TQ_ERR_INVALID_ARG otherwise.
+ */
+TQ_API tq_status tq_scale_grad(const float* w, const float* dw, const uint32_t* codes,
+                               const float* scales, int64_t n, int64_t k, int32_t g,
+                               float* dscales, void* stream);
+
 /* Hyperparameters of one AdamW step (tq_adamw_requantize). */
 typedef struct tq_adamw_hparams {
   double lr;            /* learning rate of this step (after any schedule), >= 0       */
@@ -174,6 +211,32 @@ TQ_API tq_status tq_adamw_requantize(float* w, const float* grad, float* m, floa
                                      int64_t k, int32_t g, const tq_adamw_hparams* hp,
                                      uint32_t* codes, float* scales, int32_t* zero_counts,
                                      void* stream);
+
+/*
+ * tq_adamw_requantize_with_scales — tq_adamw_requantize for the learnable-scale
+ * variant: the same AdamW update of w, m and v, then the codes and zero counts of
+ * the new w against the caller's scales exactly as tq_quantize_with_scales (pass
+ * the scales already updated for this step, e.g. by tq_adamw).
+ *   scales   fp32 [n][k/g] (device, 16-byte aligned); read only.
+ *   Other arguments, layouts and errors as tq_adamw_requantize.
+ */
+TQ_API tq_status tq_adamw_requantize_with_scales(float* w, const float* grad, float* m, float* v,
+                                                 int64_t n, int64_t k, int32_t g,
+                                                 const tq_adamw_hparams* hp, const float* scales,
+                                                 uint32_t* codes, int32_t* zero_counts,
+                                                 void* stream);
+
+/*
+ * tq_adamw — the AdamW update of tq_adamw_requantize (same operations, same
+ * rounding) over a flat fp32 array without requantization, e.g. the scales of the
+ * learnable-scale variant.
+ *   p, m, v   in/out: fp32 [count] (device, 16-byte aligned).
+ *   grad      fp32 [count] (device, 16-byte aligned).
+ *   Requires count % 16 == 0 and hp as for tq_adamw_requantize;
+ *   TQ_ERR_INVALID_ARG otherwise, before anything is launched.
+ */
+TQ_API tq_status tq_adamw(float* p, const float* grad, float* m, float* v, int64_t count,
+                          const tq_adamw_hparams* hp, void* stream);
 
 /*
  * tq_linear_fwd — W1.58A16 forward (§3.1, "W1.58A16" of the title):

@@ -20,7 +20,9 @@
 //   w  = w * (1 - lr * wd) - step_size * (m / (sqrt(v) * inv_bc2_sqrt + eps))
 // with step_size = lr / (1 - b1^t) and inv_bc2_sqrt = 1 / sqrt(1 - b2^t), the step
 // constants computed on the host in fp64 and rounded once to fp32. The new W is
-// then quantized exactly as tq_quantize does (quant_code.cuh).
+// then quantized exactly as tq_quantize does (quant_code.cuh), or against
+// caller-given scales (the learnable-scale variant), or not at all (a plain AdamW
+// step over any fp32 array of a multiple of 16 elements, e.g. those scales).
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -100,7 +102,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const int64_t e0 = st * kStageW;
         const int64_t cnt = total - e0 < kStageW ? total - e0 : kStageW;
-        const uint32_t bytes = static_cast<uint32_t>(cnt) * 4u;  // a multiple of 128 (g | k)
+        const uint32_t bytes = static_cast<uint32_t>(cnt) * 4u;  // a multiple of 64 (16 | total)
         const uint32_t dst = ring + slot * kStageBytes;
         stage_of[slot] = st;
         mbar_arrive_expect_tx(full_bar(slot), 4 * bytes);
@@ -174,27 +176,35 @@ __global__ void __launch_bounds__(kThreads, 1)
         md[q] = make_float4(mo[4 * q], mo[4 * q + 1], mo[4 * q + 2], mo[4 * q + 3]);
         vd[q] = make_float4(vo[4 * q], vo[4 * q + 1], vo[4 * q + 2], vo[4 * q + 3]);
       }
-      // requantize the new weights (as tq_quantize)
-      float sum = 0.f;
+      if (a.codes != nullptr) {
+        // requantize the new weights: against their absmean (as tq_quantize) or
+        // against the caller's scales (the learnable-scale variant)
+        float s = 0.f;
+        uint32_t word;
+        if (a.given_scale != nullptr) {
+          word = code_word_any(x, __ldg(a.given_scale + e / G), live);
+        } else {
+          float sum = 0.f;
 #pragma unroll
-      for (int q = 0; q < 4; ++q)
-        sum += (fabsf(x[4 * q]) + fabsf(x[4 * q + 1])) + (fabsf(x[4 * q + 2]) + fabsf(x[4 * q + 3]));
+          for (int q = 0; q < 4; ++q)
+            sum += (fabsf(x[4 * q]) + fabsf(x[4 * q + 1])) + (fabsf(x[4 * q + 2]) + fabsf(x[4 * q + 3]));
 #pragma unroll
-      for (int off = 1; off < kLanesPerGroup; off <<= 1) sum += __shfl_xor_sync(live, sum, off);
-      const float s = sum * kInvG;
-      const bool tiny = s < 0x1p-100f;
-      const uint32_t word = __any_sync(live, tiny)
-                                ? (tiny ? code_word<true>(x, s) : code_word<false>(x, s))
-                                : code_word<false>(x, s);
-      const unsigned gmask =
-          kLanesPerGroup == 32 ? 0xffffffffu
-                               : ((1u << kLanesPerGroup) - 1u) << (lane & ~(kLanesPerGroup - 1));
-      const int zc = static_cast<int>(
-          __reduce_add_sync(gmask, static_cast<unsigned>(16 - __popc(word & 0x55555555u))));
-      a.codes[e >> 4] = word;
-      if ((lane & (kLanesPerGroup - 1)) == 0) {
-        a.scales[e / G] = s;
-        a.zeros[e / G] = zc;
+          for (int off = 1; off < kLanesPerGroup; off <<= 1) sum += __shfl_xor_sync(live, sum, off);
+          s = sum * kInvG;
+          const bool tiny = s < 0x1p-100f;
+          word = __any_sync(live, tiny) ? (tiny ? code_word<true>(x, s) : code_word<false>(x, s))
+                                        : code_word<false>(x, s);
+        }
+        const unsigned gmask =
+            kLanesPerGroup == 32 ? 0xffffffffu
+                                 : ((1u << kLanesPerGroup) - 1u) << (lane & ~(kLanesPerGroup - 1));
+        const int zc = static_cast<int>(
+            __reduce_add_sync(gmask, static_cast<unsigned>(16 - __popc(word & 0x55555555u))));
+        a.codes[e >> 4] = word;
+        if ((lane & (kLanesPerGroup - 1)) == 0) {
+          if (a.given_scale == nullptr) a.scales[e / G] = s;
+          a.zeros[e / G] = zc;
+        }
       }
     }
     __syncwarp();

@@ -27,9 +27,12 @@ cudaError_t ensure_smem_limit(int bytes) {
 // quantize.cu ----------------------------------------------------------------
 // row_factor (fp32 [n] or null): the codes of row r are decided against the
 // threshold row_factor[r] * s instead of s (the decoupled quantizer); scales stay s.
+// given_scale (fp32 [n][k/g] or null): the codes are decided against these scales
+// (the learnable-scale variant) and scales is not written.
 cudaError_t launch_quantize(const float* w, int64_t n, int64_t k, int g, uint32_t* codes,
                             float* scales, int32_t* zeros, int* status, int num_sms,
-                            cudaStream_t stream, const float* row_factor = nullptr);
+                            cudaStream_t stream, const float* row_factor = nullptr,
+                            const float* given_scale = nullptr);
 
 // Many matrices (same group size) in one launch.
 struct QuantMat {
@@ -41,12 +44,21 @@ struct QuantMat {
   int64_t stage0;   // first stage of this matrix (set by the launcher)
   const float* row_factor;  // null, or fp32 [n]: per-row threshold factor
   int64_t k;        // row length (for row_factor)
+  const float* given_scale;  // null, or fp32 [n][k/g]: decide against these scales
+                             // (scales is then not written)
 };
 
 // dalpha[n][k/g] = sum over each group of dw * code (the decoupled quantizer's
 // magnitude gradient).
 cudaError_t launch_alpha_grad(const float* dw, const uint32_t* codes, int64_t n, int64_t k, int g,
                               float* dalpha, int num_sms, cudaStream_t stream);
+
+// dscale[n][k/g] = sum over each group of dw * (c - q [|w| < |s|]), q = w / s: the
+// gradient of a learnable scale through W^ = s * round(clip(w / s)) with the
+// rounding passed straight through.
+cudaError_t launch_scale_grad(const float* w, const float* dw, const uint32_t* codes,
+                              const float* scales, int64_t n, int64_t k, int g, float* dscale,
+                              int num_sms, cudaStream_t stream);
 
 template <int kMax>
 struct QuantBatch {
@@ -82,11 +94,12 @@ struct AdamwArgs {
   const float* grad;    // fp32 [n][k]
   float* m;             // fp32 [n][k], updated in place
   float* v;             // fp32 [n][k], updated in place
-  uint32_t* codes;      // uint32 [n][k/16] of the new w
+  uint32_t* codes;      // uint32 [n][k/16] of the new w; null: no requantization
   float* scales;        // fp32 [n][k/g]
   int32_t* zeros;       // int32 [n][k/g]
   int64_t total;        // n * k
   AdamwConst c;
+  const float* given_scale;  // null, or fp32 [n][k/g]: requantize against these
 };
 
 cudaError_t launch_adamw_requantize(const AdamwArgs& a, int g, int* status, int num_sms,

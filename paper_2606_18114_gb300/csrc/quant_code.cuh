@@ -50,4 +50,20 @@ __device__ __forceinline__ uint32_t code_word(const float (&x)[16], float s) {
   return nz | (neg & (nz << 1));
 }
 
+// Code word against a caller-given scale of either sign (the learnable-scale
+// variant): c = round(clip(w / s)). For s < 0 the fp32 quotient of the negated
+// operands is the same number, so the word is that of -w against -s; scales below
+// 2^-100 (zero, denormal) or NaN-free tiny values take the division. Every lane in
+// `live` must call it.
+__device__ __forceinline__ uint32_t code_word_any(const float (&x)[16], float s, unsigned live) {
+  const bool flip = s < 0.f;
+  const float t = flip ? -s : s;
+  float y[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) y[j] = flip ? -x[j] : x[j];
+  const bool tiny = t < 0x1p-100f;
+  return __any_sync(live, tiny) ? (tiny ? code_word<true>(y, t) : code_word<false>(y, t))
+                                : code_word<false>(y, t);
+}
+
 }  // namespace tq

@@ -176,22 +176,30 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       float4 v[4];
 #pragma unroll
       for (int j = 0; j < 4; ++j) v[j] = src[j];
-      float sum = 0.f;
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        sum += (fabsf(v[j].x) + fabsf(v[j].y)) + (fabsf(v[j].z) + fabsf(v[j].w));
-#pragma unroll
-      for (int off = 1; off < kLanesPerGroup; off <<= 1) sum += __shfl_xor_sync(live, sum, off);
-      const float s = sum * kInvG;  // s = (1/g) * sum |w|
-      // the decoupled quantizer decides against tau = f_row * s (one fp32 product)
-      const float tau = mt.row_factor == nullptr ? s : __fmul_rn(s, mt.row_factor[e / mt.k]);
       const float x[16] = {v[0].x, v[0].y, v[0].z, v[0].w, v[1].x, v[1].y, v[1].z, v[1].w,
                            v[2].x, v[2].y, v[2].z, v[2].w, v[3].x, v[3].y, v[3].z, v[3].w};
-      // thresholds below 2^-100 (all-zero or denormal groups) take the division
-      const bool tiny = tau < 0x1p-100f;
-      const uint32_t word = __any_sync(live, tiny)
-                                ? (tiny ? code_word<true>(x, tau) : code_word<false>(x, tau))
-                                : code_word<false>(x, tau);
+      const bool given = mt.given_scale != nullptr;  // uniform: one matrix per stage
+      float s = 0.f;
+      uint32_t word;
+      if (given) {
+        // the learnable-scale variant: the caller's scale decides, of either sign
+        word = code_word_any(x, __ldg(mt.given_scale + e / G), live);
+      } else {
+        float sum = 0.f;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          sum += (fabsf(v[j].x) + fabsf(v[j].y)) + (fabsf(v[j].z) + fabsf(v[j].w));
+#pragma unroll
+        for (int off = 1; off < kLanesPerGroup; off <<= 1) sum += __shfl_xor_sync(live, sum, off);
+        s = sum * kInvG;  // s = (1/g) * sum |w|
+        // the decoupled quantizer decides against tau = f_row * s (one fp32 product)
+        const float tau = mt.row_factor == nullptr ? s : __fmul_rn(s, mt.row_factor[e / mt.k]);
+        // thresholds below 2^-100 (all-zero or denormal groups) take the division
+        const bool tiny = tau < 0x1p-100f;
+        word = __any_sync(live, tiny)
+                   ? (tiny ? code_word<true>(x, tau) : code_word<false>(x, tau))
+                   : code_word<false>(x, tau);
+      }
       const unsigned gmask =
           kLanesPerGroup == 32 ? 0xffffffffu
                                : ((1u << kLanesPerGroup) - 1u) << (lane & ~(kLanesPerGroup - 1));
@@ -199,7 +207,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
           __reduce_add_sync(gmask, static_cast<unsigned>(16 - __popc(word & 0x55555555u))));
       mt.codes[e >> 4] = word;
       if ((lane & (kLanesPerGroup - 1)) == 0) {
-        mt.scales[e / G] = s;
+        if (!given) mt.scales[e / G] = s;
         mt.zeros[e / G] = zc;
       }
     }
@@ -381,6 +389,85 @@ cudaError_t launch_alpha_grad(const float* dw, const uint32_t* codes, int64_t n,
   }
 }
 
+namespace {
+
+// dscale of the learnable-scale variant: a lane per code word; per group the sums
+// A = sum dw * c and B = sum over |w| < |s| of dw * w, reduced over the group's
+// lanes; dscale = A - B / s (B is 0 when s is 0: no |w| is below it).
+template <int G>
+__global__ void __launch_bounds__(256) scale_grad_kernel(const float* __restrict__ w,
+                                                         const float* __restrict__ dw,
+                                                         const uint32_t* __restrict__ codes,
+                                                         const float* __restrict__ scales,
+                                                         int64_t words, float* __restrict__ ds) {
+  constexpr int kLanesPerGroup = G / 16;
+  const int lane = threadIdx.x & 31;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31);
+       base < words; base += stride) {
+    const int64_t wi = base + lane;
+    if (wi >= words) continue;  // whole groups: the lanes of a group agree
+    const int64_t gi = wi / kLanesPerGroup;
+    const uint32_t c = __ldg(codes + wi);
+    const float s = __ldg(scales + gi);
+    const float as = fabsf(s);
+    const float4* pd = reinterpret_cast<const float4*>(dw + wi * 16);
+    const float4* pw = reinterpret_cast<const float4*>(w + wi * 16);
+    float a = 0.f, b = 0.f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 d4 = __ldg(pd + q);
+      const float4 w4 = __ldg(pw + q);
+      const float d[4] = {d4.x, d4.y, d4.z, d4.w};
+      const float x[4] = {w4.x, w4.y, w4.z, w4.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int j = 4 * q + i;
+        const int bit = 16 * (j & 1) + 2 * (j >> 1);  // code j of the word (include/tq.h)
+        const float t = (c >> (bit + 1)) & 1u ? -d[i] : d[i];
+        a += (c >> bit) & 1u ? t : 0.f;
+        b += fabsf(x[i]) < as ? d[i] * x[i] : 0.f;
+      }
+    }
+    const unsigned gmask =
+        kLanesPerGroup == 32 ? 0xffffffffu
+                             : ((1u << kLanesPerGroup) - 1u) << (lane & ~(kLanesPerGroup - 1));
+#pragma unroll
+    for (int off = 1; off < kLanesPerGroup; off <<= 1) {
+      a += __shfl_xor_sync(gmask, a, off);
+      b += __shfl_xor_sync(gmask, b, off);
+    }
+    if ((lane & (kLanesPerGroup - 1)) == 0) ds[gi] = b == 0.f ? a : a - __fdiv_rn(b, s);
+  }
+}
+
+template <int G>
+cudaError_t launch_sg(const float* w, const float* dw, const uint32_t* codes, const float* scales,
+                      int64_t words, float* ds, int num_sms, cudaStream_t stream) {
+  const int64_t need = (words + 255) / 256;
+  const int64_t cap = static_cast<int64_t>(num_sms) * 8;
+  scale_grad_kernel<G><<<static_cast<unsigned>(need < cap ? need : cap), 256, 0, stream>>>(
+      w, dw, codes, scales, words, ds);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_scale_grad(const float* w, const float* dw, const uint32_t* codes,
+                              const float* scales, int64_t n, int64_t k, int g, float* dscale,
+                              int num_sms, cudaStream_t stream) {
+  const int64_t words = n * k / 16;
+  if (words <= 0) return cudaSuccess;
+  switch (g) {
+    case 32: return launch_sg<32>(w, dw, codes, scales, words, dscale, num_sms, stream);
+    case 64: return launch_sg<64>(w, dw, codes, scales, words, dscale, num_sms, stream);
+    case 128: return launch_sg<128>(w, dw, codes, scales, words, dscale, num_sms, stream);
+    case 256: return launch_sg<256>(w, dw, codes, scales, words, dscale, num_sms, stream);
+    case 512: return launch_sg<512>(w, dw, codes, scales, words, dscale, num_sms, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
 cudaError_t launch_transpose_codes(const uint32_t* codes, int64_t n, int64_t k, uint32_t* codes_t,
                                    cudaStream_t stream) {
   const int64_t ldt = 4 * ((n + 63) / 64);
@@ -391,9 +478,10 @@ cudaError_t launch_transpose_codes(const uint32_t* codes, int64_t n, int64_t k, 
 
 cudaError_t launch_quantize(const float* w, int64_t n, int64_t k, int g, uint32_t* codes,
                             float* scales, int32_t* zeros, int* status, int num_sms,
-                            cudaStream_t stream, const float* row_factor) {
+                            cudaStream_t stream, const float* row_factor,
+                            const float* given_scale) {
   QuantBatch<1> b{};
-  b.mats[0] = QuantMat{w, codes, scales, zeros, n * k, 0, row_factor, k};
+  b.mats[0] = QuantMat{w, codes, scales, zeros, n * k, 0, row_factor, k, given_scale};
   b.count = 1;
   b.nstages = (n * k + kStageW - 1) / kStageW;
   return launch_g<1>(b, g, status, num_sms, stream);

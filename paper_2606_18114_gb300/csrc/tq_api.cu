@@ -383,6 +383,44 @@ TQ_API tq_status tq_alpha_grad(const float* dw, const uint32_t* codes, int64_t n
   return e == cudaSuccess ? TQ_OK : cuda_fail(e, "alpha_grad launch");
 }
 
+TQ_API tq_status tq_quantize_with_scales(const float* w, int64_t n, int64_t k, int32_t g,
+                                         const float* scales, uint32_t* codes,
+                                         int32_t* zero_counts, void* stream) {
+  g_err[0] = 0;
+  // the scales are an input here; the absmean check of tq_quantize covers the rest
+  TQ_TRY(check_quantize_args(w, n, k, g, codes, scales, zero_counts));
+  if (n == 0 || k == 0) return TQ_OK;
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaError_t e = tq::launch_quantize(w, n, k, g, codes, nullptr, zero_counts, dev->status,
+                                      dev->num_sms, static_cast<cudaStream_t>(stream), nullptr,
+                                      scales);
+  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "quantize launch");
+}
+
+TQ_API tq_status tq_scale_grad(const float* w, const float* dw, const uint32_t* codes,
+                               const float* scales, int64_t n, int64_t k, int32_t g,
+                               float* dscales, void* stream) {
+  g_err[0] = 0;
+  if (n < 0 || k < 0) return fail(TQ_ERR_INVALID_ARG, "negative size");
+  if (log2_group(g) < 0) return fail(TQ_ERR_INVALID_ARG, "group size %d not in {32..512}", g);
+  if (k % g != 0) return fail(TQ_ERR_INVALID_ARG, "k=%lld is not a multiple of g=%d", (long long)k, g);
+  if (n == 0 || k == 0) return TQ_OK;
+  if (n > INT64_MAX / k) return fail(TQ_ERR_INVALID_ARG, "n*k overflows");
+  TQ_TRY(check_ptr(w, "w"));
+  TQ_TRY(check_ptr(dw, "dw"));
+  TQ_TRY(check_ptr(codes, "codes"));
+  if (scales == nullptr || (reinterpret_cast<uintptr_t>(scales) & 3) != 0)
+    return fail(TQ_ERR_INVALID_ARG, "scales is NULL or not 4-byte aligned");
+  if (dscales == nullptr || (reinterpret_cast<uintptr_t>(dscales) & 3) != 0)
+    return fail(TQ_ERR_INVALID_ARG, "dscales is NULL or not 4-byte aligned");
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaError_t e = tq::launch_scale_grad(w, dw, codes, scales, n, k, g, dscales, dev->num_sms,
+                                        static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "scale_grad launch");
+}
+
 TQ_API tq_status tq_quantize_batched(const tq_quant_desc* descs, int32_t count, int32_t g,
                                      void* stream) {
   g_err[0] = 0;
@@ -411,12 +449,10 @@ TQ_API tq_status tq_quantize_batched(const tq_quant_desc* descs, int32_t count, 
   return e == cudaSuccess ? TQ_OK : cuda_fail(e, "quantize launch");
 }
 
-TQ_API tq_status tq_adamw_requantize(float* w, const float* grad, float* m, float* v, int64_t n,
-                                     int64_t k, int32_t g, const tq_adamw_hparams* hp,
-                                     uint32_t* codes, float* scales, int32_t* zero_counts,
-                                     void* stream) {
-  g_err[0] = 0;
-  TQ_TRY(check_quantize_args(w, n, k, g, codes, scales, zero_counts));
+namespace {
+// AdamW hyperparameters checked and turned into the kernel's fp32 step constants
+// (computed in fp64, rounded once).
+tq_status adamw_const(const tq_adamw_hparams* hp, tq::AdamwConst* c) {
   if (hp == nullptr) return fail(TQ_ERR_INVALID_ARG, "hparams is NULL");
   if (hp->step < 1) return fail(TQ_ERR_INVALID_ARG, "step %lld < 1", (long long)hp->step);
   const double lr = hp->lr, b1 = hp->beta1, b2 = hp->beta2, eps = hp->eps;
@@ -424,11 +460,40 @@ TQ_API tq_status tq_adamw_requantize(float* w, const float* grad, float* m, floa
   if (!(lr >= 0 && lr < 1e30) || !(b1 >= 0 && b1 < 1) || !(b2 >= 0 && b2 < 1) ||
       !(eps > 0 && eps < 1e30) || !(wd >= 0 && wd < 1e30) || !(gs >= 0 && gs < 1e30))
     return fail(TQ_ERR_INVALID_ARG, "hyperparameters out of range");
+  const double t = static_cast<double>(hp->step);
+  c->b1 = static_cast<float>(b1);
+  c->omb1 = static_cast<float>(1.0 - b1);
+  c->b2 = static_cast<float>(b2);
+  c->omb2 = static_cast<float>(1.0 - b2);
+  c->decay = static_cast<float>(1.0 - lr * wd);
+  c->step_size = static_cast<float>(lr / (1.0 - pow(b1, t)));
+  c->inv_bc2_sqrt = static_cast<float>(1.0 / sqrt(1.0 - pow(b2, t)));
+  c->eps = static_cast<float>(eps);
+  c->grad_scale = static_cast<float>(gs);
+  return TQ_OK;
+}
+
+tq_status adamw_launch(tq::AdamwArgs& a, int32_t g, void* stream) {
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaError_t e = tq::launch_adamw_requantize(a, g, dev->status, dev->num_sms,
+                                              static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "adamw launch");
+}
+}  // namespace
+
+TQ_API tq_status tq_adamw_requantize(float* w, const float* grad, float* m, float* v, int64_t n,
+                                     int64_t k, int32_t g, const tq_adamw_hparams* hp,
+                                     uint32_t* codes, float* scales, int32_t* zero_counts,
+                                     void* stream) {
+  g_err[0] = 0;
+  TQ_TRY(check_quantize_args(w, n, k, g, codes, scales, zero_counts));
+  tq::AdamwArgs a{};
+  TQ_TRY(adamw_const(hp, &a.c));
   if (n == 0 || k == 0) return TQ_OK;
   TQ_TRY(check_ptr(grad, "grad"));
   TQ_TRY(check_ptr(m, "m"));
   TQ_TRY(check_ptr(v, "v"));
-  tq::AdamwArgs a{};
   a.w = w;
   a.grad = grad;
   a.m = m;
@@ -437,22 +502,51 @@ TQ_API tq_status tq_adamw_requantize(float* w, const float* grad, float* m, floa
   a.scales = scales;
   a.zeros = zero_counts;
   a.total = n * k;
-  // step constants: fp64, rounded once to fp32
-  const double t = static_cast<double>(hp->step);
-  a.c.b1 = static_cast<float>(b1);
-  a.c.omb1 = static_cast<float>(1.0 - b1);
-  a.c.b2 = static_cast<float>(b2);
-  a.c.omb2 = static_cast<float>(1.0 - b2);
-  a.c.decay = static_cast<float>(1.0 - lr * wd);
-  a.c.step_size = static_cast<float>(lr / (1.0 - pow(b1, t)));
-  a.c.inv_bc2_sqrt = static_cast<float>(1.0 / sqrt(1.0 - pow(b2, t)));
-  a.c.eps = static_cast<float>(eps);
-  a.c.grad_scale = static_cast<float>(gs);
-  const DeviceInfo* dev = nullptr;
-  TQ_TRY(device_info(&dev));
-  cudaError_t e = tq::launch_adamw_requantize(a, g, dev->status, dev->num_sms,
-                                              static_cast<cudaStream_t>(stream));
-  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "adamw launch");
+  return adamw_launch(a, g, stream);
+}
+
+TQ_API tq_status tq_adamw_requantize_with_scales(float* w, const float* grad, float* m, float* v,
+                                                 int64_t n, int64_t k, int32_t g,
+                                                 const tq_adamw_hparams* hp, const float* scales,
+                                                 uint32_t* codes, int32_t* zero_counts,
+                                                 void* stream) {
+  g_err[0] = 0;
+  TQ_TRY(check_quantize_args(w, n, k, g, codes, scales, zero_counts));
+  tq::AdamwArgs a{};
+  TQ_TRY(adamw_const(hp, &a.c));
+  if (n == 0 || k == 0) return TQ_OK;
+  TQ_TRY(check_ptr(grad, "grad"));
+  TQ_TRY(check_ptr(m, "m"));
+  TQ_TRY(check_ptr(v, "v"));
+  a.w = w;
+  a.grad = grad;
+  a.m = m;
+  a.v = v;
+  a.codes = codes;
+  a.zeros = zero_counts;
+  a.given_scale = scales;
+  a.total = n * k;
+  return adamw_launch(a, g, stream);
+}
+
+TQ_API tq_status tq_adamw(float* p, const float* grad, float* m, float* v, int64_t count,
+                          const tq_adamw_hparams* hp, void* stream) {
+  g_err[0] = 0;
+  if (count < 0) return fail(TQ_ERR_INVALID_ARG, "negative count");
+  if (count % 16 != 0) return fail(TQ_ERR_INVALID_ARG, "count=%lld is not a multiple of 16", (long long)count);
+  tq::AdamwArgs a{};
+  TQ_TRY(adamw_const(hp, &a.c));
+  if (count == 0) return TQ_OK;
+  TQ_TRY(check_ptr(p, "p"));
+  TQ_TRY(check_ptr(grad, "grad"));
+  TQ_TRY(check_ptr(m, "m"));
+  TQ_TRY(check_ptr(v, "v"));
+  a.w = p;
+  a.grad = grad;
+  a.m = m;
+  a.v = v;
+  a.total = count;  // codes == nullptr: no requantization
+  return adamw_launch(a, 128, stream);
 }
 
 TQ_API tq_status tq_linear_fwd(const void* x, int64_t m, int64_t k, const uint32_t* codes,

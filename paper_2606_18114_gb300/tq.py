@@ -28,6 +28,10 @@ __all__ = [
     "adamw_requantize",
     "quantize_decoupled",
     "alpha_grad",
+    "quantize_with_scales",
+    "scale_grad",
+    "adamw_requantize_with_scales",
+    "adamw",
     "AdamwHparams",
     "version",
     "OUT_F32",
@@ -44,7 +48,8 @@ STATUS = {0: "TQ_OK", 1: "TQ_ERR_INVALID_ARG", 2: "TQ_ERR_UNSUPPORTED", 3: "TQ_E
 EXPORTS = ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
            "tq_linear_bwd_noalloc", "tq_codes_transpose", "tq_linear_fwd_batched",
            "tq_adamw_requantize", "tq_quantize_decoupled", "tq_alpha_grad",
-           "tq_device_status", "tq_last_error", "tq_version")
+           "tq_quantize_with_scales", "tq_scale_grad", "tq_adamw_requantize_with_scales",
+           "tq_adamw", "tq_device_status", "tq_last_error", "tq_version")
 
 _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtq.so")
 _lib = None
@@ -116,6 +121,11 @@ def load(path: Optional[str] = None):
     lib.tq_alpha_grad.argtypes = [vp, vp, i64, i64, i32, vp, vp]
     lib.tq_adamw_requantize.argtypes = [vp, vp, vp, vp, i64, i64, i32, ctypes.POINTER(AdamwHparams),
                                         vp, vp, vp, vp]
+    lib.tq_quantize_with_scales.argtypes = [vp, i64, i64, i32, vp, vp, vp, vp]
+    lib.tq_scale_grad.argtypes = [vp, vp, vp, vp, i64, i64, i32, vp, vp]
+    lib.tq_adamw_requantize_with_scales.argtypes = [vp, vp, vp, vp, i64, i64, i32,
+                                                    ctypes.POINTER(AdamwHparams), vp, vp, vp, vp]
+    lib.tq_adamw.argtypes = [vp, vp, vp, vp, i64, ctypes.POINTER(AdamwHparams), vp]
     for name in ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
                  "tq_linear_bwd_noalloc", "tq_codes_transpose", "tq_linear_fwd_batched",
                  "tq_device_status"):
@@ -222,6 +232,61 @@ def alpha_grad(dw: torch.Tensor, codes: torch.Tensor, g: int, out: Optional[torc
         out = torch.empty((n, k // g), dtype=torch.float32, device=dw.device)
     _check(load().tq_alpha_grad(_ptr(dw), _ptr(codes), n, k, g, _ptr(out), _stream(stream)))
     return out
+
+
+def quantize_with_scales(w: torch.Tensor, g: int, scales: torch.Tensor, out=None, stream=None):
+    """The learnable-scale variant's quantizer: codes against the given per-group
+    ``scales`` (fp32 ``[N, K/g]``, any sign). Returns ``(codes, zero_counts)``."""
+    n, k = w.shape
+    if out is None:
+        codes = torch.empty((n, k // 16), dtype=torch.int32, device=w.device)
+        zeros = torch.empty((n, k // g), dtype=torch.int32, device=w.device)
+    else:
+        codes, zeros = out
+    _check(load().tq_quantize_with_scales(_ptr(w), n, k, g, _ptr(scales), _ptr(codes),
+                                          _ptr(zeros), _stream(stream)))
+    return codes, zeros
+
+
+def scale_grad(w: torch.Tensor, dw: torch.Tensor, codes: torch.Tensor, scales: torch.Tensor,
+               g: int, out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Gradient of the learnable scales (include/tq.h, tq_scale_grad)."""
+    n, k = w.shape
+    if out is None:
+        out = torch.empty((n, k // g), dtype=torch.float32, device=w.device)
+    _check(load().tq_scale_grad(_ptr(w), _ptr(dw), _ptr(codes), _ptr(scales), n, k, g, _ptr(out),
+                                _stream(stream)))
+    return out
+
+
+def adamw_requantize_with_scales(w: torch.Tensor, grad: torch.Tensor, m: torch.Tensor,
+                                 v: torch.Tensor, g: int, scales: torch.Tensor, lr: float,
+                                 step: int, beta1: float = 0.9, beta2: float = 0.95,
+                                 eps: float = 1e-8, weight_decay: float = 0.01,
+                                 grad_scale: float = 1.0, out=None, stream=None):
+    """:func:`adamw_requantize` with the codes of the new ``w`` decided against the
+    given ``scales``. Returns ``(codes, zero_counts)``."""
+    n, k = w.shape
+    if out is None:
+        codes = torch.empty((n, k // 16), dtype=torch.int32, device=w.device)
+        zeros = torch.empty((n, k // g), dtype=torch.int32, device=w.device)
+    else:
+        codes, zeros = out
+    hp = AdamwHparams(lr, beta1, beta2, eps, weight_decay, grad_scale, step)
+    _check(load().tq_adamw_requantize_with_scales(_ptr(w), _ptr(grad), _ptr(m), _ptr(v), n, k, g,
+                                                  ctypes.byref(hp), _ptr(scales), _ptr(codes),
+                                                  _ptr(zeros), _stream(stream)))
+    return codes, zeros
+
+
+def adamw(p: torch.Tensor, grad: torch.Tensor, m: torch.Tensor, v: torch.Tensor, lr: float,
+          step: int, beta1: float = 0.9, beta2: float = 0.95, eps: float = 1e-8,
+          weight_decay: float = 0.01, grad_scale: float = 1.0, stream=None) -> None:
+    """One AdamW step on a flat fp32 array ``p`` (numel a multiple of 16); ``p``, ``m``
+    and ``v`` are updated in place."""
+    hp = AdamwHparams(lr, beta1, beta2, eps, weight_decay, grad_scale, step)
+    _check(load().tq_adamw(_ptr(p), _ptr(grad), _ptr(m), _ptr(v), p.numel(), ctypes.byref(hp),
+                           _stream(stream)))
 
 
 def quant_batch(items: Sequence[tuple]):

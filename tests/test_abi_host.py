@@ -189,6 +189,36 @@ def test_decoupled_and_alpha_grad_reject_before_launch(lib):
     assert ag(FAKE, FAKE, 0, 256, 128, FAKE, None) == 0                   # empty
 
 
+def test_learnable_scale_entries_reject_before_launch(lib):
+    from paper_2606_18114_gb300.tq import AdamwHparams
+    import ctypes
+    hp = ctypes.byref(AdamwHparams(2.5e-4, 0.9, 0.95, 1e-8, 0.01, 1.0, 1))
+    q, sg = lib.tq_quantize_with_scales, lib.tq_scale_grad
+    assert q(FAKE, 8, 96, 64, FAKE, FAKE, FAKE, None) == 1                # k % g
+    assert q(FAKE, 8, 256, 48, FAKE, FAKE, FAKE, None) == 1               # group size
+    assert q(FAKE, 8, 256, 128, None, FAKE, FAKE, None) == 1              # null scales
+    assert q(FAKE, 8, 256, 128, MIS, FAKE, FAKE, None) == 1               # misaligned scales
+    assert q(FAKE, 0, 256, 128, FAKE, FAKE, FAKE, None) == 0              # empty
+    assert sg(FAKE, FAKE, FAKE, FAKE, 8, 96, 64, FAKE, None) == 1         # k % g
+    assert sg(FAKE, FAKE, FAKE, FAKE, 8, 256, 16, FAKE, None) == 1        # group size
+    assert sg(FAKE, MIS, FAKE, FAKE, 8, 256, 128, FAKE, None) == 1        # misaligned dw
+    assert sg(FAKE, FAKE, FAKE, None, 8, 256, 128, FAKE, None) == 1       # null scales
+    assert sg(FAKE, FAKE, FAKE, FAKE, 8, 256, 128, None, None) == 1       # null dscales
+    assert b"dscales" in lib.tq_last_error()
+    assert sg(FAKE, FAKE, FAKE, FAKE, 0, 256, 128, FAKE, None) == 0       # empty
+    a = lib.tq_adamw_requantize_with_scales
+    assert a(FAKE, FAKE, FAKE, FAKE, 8, 256, 128, None, FAKE, FAKE, FAKE, None) == 1  # no hparams
+    assert a(FAKE, FAKE, FAKE, FAKE, 8, 256, 128, hp, None, FAKE, FAKE, None) == 1    # null scales
+    assert a(FAKE, FAKE, FAKE, FAKE, 8, 96, 64, hp, FAKE, FAKE, FAKE, None) == 1      # k % g
+    assert a(FAKE, FAKE, FAKE, FAKE, 0, 256, 128, hp, FAKE, FAKE, FAKE, None) == 0    # empty
+    p = lib.tq_adamw
+    assert p(FAKE, FAKE, FAKE, FAKE, 24, hp, None) == 1                   # count % 16
+    assert p(FAKE, FAKE, FAKE, FAKE, -16, hp, None) == 1                  # negative count
+    assert p(FAKE, FAKE, FAKE, FAKE, 32, None, None) == 1                 # no hparams
+    assert p(FAKE, MIS, FAKE, FAKE, 32, hp, None) == 1                    # misaligned grad
+    assert p(FAKE, FAKE, FAKE, FAKE, 0, hp, None) == 0                    # empty
+
+
 def test_activation_flag_checked(lib):
     """The output-type word takes TQ_IN_F16 and nothing else beyond the output type;
     a batched decode takes one activation type."""
