@@ -556,6 +556,59 @@ def decoupled_sweep(tq, steps, warmup):
     return res
 
 
+def learnable_sweep(tq, steps, warmup):
+    """The learnable-scale variant on in_proj: codes against given scales, the
+    scale gradient, and the fused AdamW step with requantization against given
+    scales; then the zero ratio of both scale parameterizations over a synthetic
+    teacher-student run (paper_2606_18114_gb300.qat) on the out_proj shape."""
+    from paper_2606_18114_gb300 import qat
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(43)
+    pk, _ = peaks()
+    n, k = IN_PROJ
+    w = torch.randn((n, k), generator=gen, device="cuda") * 0.02
+    dw = torch.randn((n, k), generator=gen, device="cuda") * 1e-3
+    m, v = torch.zeros_like(w), torch.randn((n, k), generator=gen, device="cuda").abs() * 1e-7
+    codes, s, z = tq.quantize(w, G)
+    s.mul_(1.1)
+    ds = torch.empty_like(s)
+    res = {}
+    for label, fn, nbytes in (
+            ("quantize_with_scales", lambda: tq.quantize_with_scales(w, G, s, out=(codes, z)),
+             n * k * 4 + n * k // 4 + 8 * n * k // G),
+            ("scale_grad", lambda: tq.scale_grad(w, dw, codes, s, G, out=ds),
+             2 * n * k * 4 + n * k // 4 + 8 * n * k // G),
+            ("adamw_requantize_with_scales",
+             lambda: tq.adamw_requantize_with_scales(w, dw, m, v, G, s, lr=1e-9, step=1,
+                                                     out=(codes, z)),
+             28 * n * k + n * k // 4 + 8 * n * k // G)):
+        for _ in range(warmup):
+            fn()
+        torch.cuda.synchronize()
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record()
+        for _ in range(steps):
+            fn()
+        t1.record()
+        torch.cuda.synchronize()
+        ms = t0.elapsed_time(t1) / steps
+        res[label] = {"us": round(ms * 1e3, 2), "GB/s": round(nbytes / ms / 1e6, 1),
+                      "frac": round(nbytes / ms / 1e6 / pk["hbm_gbs"], 4), "bytes": nbytes}
+    tq.device_status()
+    on, ok = OUT_PROJ
+    track = {}
+    for label, learnable in (("fixed_absmean", False), ("learnable_scale", True)):
+        rows = qat.track_zero_ratio(tq, on, ok, 1024, G, 2000, learnable, seed=5, every=400)
+        track[label] = [{kk: (round(vv, 7) if kk == "loss" else vv) for kk, vv in r.items()}
+                        for r in rows]
+    res["zero_ratio_tracking"] = {
+        "task": f"teacher-student regression, W [{on}, {ok}] g={G}, 1024 tokens per step, "
+                "AdamW lr 2.5e-4, student from the teacher's weights",
+        **track}
+    return res
+
+
 def cublas_context(tq):
     """cuBLAS bf16 dense GEMM of the forward's shape (Y = X W^T, 16384 x 8512 x 2048):
     context for the tensor-core fraction, not part of the path."""
@@ -798,6 +851,7 @@ def main():
             "sweep_48_layers": g_sweep(tq),
             "adamw_requantize_g128": adamw_sweep(tq, 5, 2),
             "decoupled_in_proj": decoupled_sweep(tq, 20, 3),
+            "learnable_scale_in_proj": learnable_sweep(tq, 20, 3),
             "cublas_bf16_fwd_shape": cublas_context(tq),
             "hbm_peak_gbs": pk["hbm_gbs"],
         }

@@ -172,3 +172,19 @@ def test_learnable_qat_step(tq):
         w, dwg, np.zeros_like(w), np.zeros_like(w), g, cst, s1)
     assert np.array_equal(to_np(wd).view(np.uint32), w1.view(np.uint32))
     _check_codes(codes1, z1, ref_codes1, ref_z1)
+
+
+def test_zero_ratio_tracking_runs(tq):
+    """The synthetic tracking driver: both parameterizations start from the same
+    codes (the absmean of the teacher's weights, ~31 % zeros for Gaussian weights),
+    stay finite, and only the learnable run moves its scales off the absmean."""
+    from paper_2606_18114_gb300 import qat
+    a = qat.track_zero_ratio(tq, 256, 512, 256, 128, 20, learnable=False, seed=3, every=10)
+    b = qat.track_zero_ratio(tq, 256, 512, 256, 128, 20, learnable=True, seed=3, every=10)
+    assert [r["step"] for r in a] == [0, 10, 20] == [r["step"] for r in b]
+    assert a[0]["zero_ratio"] == b[0]["zero_ratio"] and a[0]["loss"] == b[0]["loss"]
+    assert abs(a[0]["zero_ratio"] - 0.31) < 0.02
+    for r in a + b:
+        assert 0.0 <= r["zero_ratio"] <= 1.0 and np.isfinite(r["loss"])
+    assert all(abs(r["scale_ratio"] - 1.0) < 1e-3 for r in a)
+    assert b[-1]["scale_ratio"] != b[0]["scale_ratio"]
