@@ -188,13 +188,15 @@ struct DwArgs {
   int32_t in_f16;  // 1: fp16 dy and x (else bf16)
 };
 
-constexpr int kDwTileK = 128;  // lanes: input features
+constexpr int kDwTileK = 128;  // lanes: input features (one CTA of a pair)
+constexpr int kDwPairK = 2 * kDwTileK;  // input features of a CTA pair's tile
 constexpr int kDwTileN = 256;  // columns: output features
-constexpr int kDwMaxCtas = 160;  // grid cap (stream-K workspace: two tiles per CTA)
+constexpr int kDwMaxCtas = 160;  // grid cap (stream-K workspace: two half-tiles per CTA)
 size_t dw_smem_bytes();
 
 // tmap_x: bf16 x [m][k] box {64, 64}; tmap_dy: bf16 dy [m][n] box {64, 64};
-// both with the 128-byte swizzle. Persistent: min(tiles, num_sms) CTAs.
+// both with the 128-byte swizzle. Persistent: clusters of two CTAs (one pair per
+// two SMs), min(tiles, resident pairs) pairs.
 cudaError_t launch_dw_gemm(const CUtensorMap& tmap_x, const CUtensorMap& tmap_dy,
                            const DwArgs& args, int num_sms, cudaStream_t stream);
 
