@@ -806,15 +806,20 @@ def main():
             kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "GB/s",
                            "frac": round(ach / pk["hbm_gbs"], 4)}
         else:
+            # timed inside the long step loop, at the power cap: the sustained peak
+            # is the denominator; the burst fraction is kept beside it
             ach = gemm_flops / (t * 1e-3) / 1e12
             kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "TFLOP/s",
-                           "frac": round(ach / pk["bf16_tflops"], 4)}
+                           "frac": round(ach / pk["bf16_tflops_sustained"], 4),
+                           "frac_of_burst": round(ach / pk["bf16_tflops"], 4)}
     dom = max((n for n, _, _ in KERNELS if n not in ("quantize", "transpose")), key=lambda n: per[n])
     dom_files = dict((n, f) for n, f, _ in KERNELS)[dom]
     roof = {"kernel": dom, "bound": "tensor", "achieved": kinfo[dom]["achieved"],
-            "peak": pk["bf16_tflops"], "unit": "TFLOP/s", "frac": kinfo[dom]["frac"],
+            "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s", "frac": kinfo[dom]["frac"],
             "traffic": recorded_traffic(dom, dom_files),
-            "peak_kind": f"{pk_kind} bf16 dense (burst)",
+            "peak_kind": f"{pk_kind} bf16 dense, sustained (the kernel is timed inside the "
+                         f"{args.steps}-step loop, at the power cap)",
+            "frac_of_burst": kinfo[dom]["frac_of_burst"], "burst_peak": pk["bf16_tflops"],
             "algorithmic_per_launch": gemm_flops}
 
     e2e_steps = max(5, args.steps // 10)
