@@ -49,7 +49,11 @@ __device__ uint32_t g_asched[kSchedSlots][2];  // {next dynamic stage, CTAs done
 
 __device__ __forceinline__ float4 ld4(const uint8_t* p) { return *reinterpret_cast<const float4*>(p); }
 
-template <int G>
+// kMode: what follows the update — the absmean requantization (kAbsmean), codes
+// against the caller's scales (kGivenScales), or nothing (kPlain).
+enum : int { kAbsmean = 0, kGivenScales = 1, kPlain = 2 };
+
+template <int G, int kMode>
 __global__ void __launch_bounds__(kThreads, 1)
     adamw_requantize_kernel(const AdamwArgs a, uint32_t* sched, int* status) {
   constexpr int kLanesPerGroup = G / 16;
@@ -176,12 +180,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         md[q] = make_float4(mo[4 * q], mo[4 * q + 1], mo[4 * q + 2], mo[4 * q + 3]);
         vd[q] = make_float4(vo[4 * q], vo[4 * q + 1], vo[4 * q + 2], vo[4 * q + 3]);
       }
-      if (a.codes != nullptr) {
+      if constexpr (kMode != kPlain) {
         // requantize the new weights: against their absmean (as tq_quantize) or
         // against the caller's scales (the learnable-scale variant)
         float s = 0.f;
         uint32_t word;
-        if (a.given_scale != nullptr) {
+        if constexpr (kMode == kGivenScales) {
           word = code_word_any(x, __ldg(a.given_scale + e / G), live);
         } else {
           float sum = 0.f;
@@ -202,7 +206,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             __reduce_add_sync(gmask, static_cast<unsigned>(16 - __popc(word & 0x55555555u))));
         a.codes[e >> 4] = word;
         if ((lane & (kLanesPerGroup - 1)) == 0) {
-          if (a.given_scale == nullptr) a.scales[e / G] = s;
+          if (kMode == kAbsmean) a.scales[e / G] = s;
           a.zeros[e / G] = zc;
         }
       }
@@ -230,35 +234,42 @@ uint32_t* asched_base() {
   return static_cast<uint32_t*>(p);
 }
 
-template <int G>
+template <int G, int kMode>
 cudaError_t launch(const AdamwArgs& a, int* status, int num_sms, cudaStream_t stream) {
   static std::atomic<uint32_t> seq{0};
   const int64_t nstages = (a.total + kStageW - 1) / kStageW;
   if (nstages <= 0) return cudaSuccess;
   if (nstages >= (int64_t{1} << 31)) return cudaErrorInvalidValue;
   const int64_t blocks = nstages < num_sms ? nstages : num_sms;
-  cudaError_t e = ensure_smem_limit<adamw_requantize_kernel<G>>(kSmemBytes);
+  cudaError_t e = ensure_smem_limit<adamw_requantize_kernel<G, kMode>>(kSmemBytes);
   if (e != cudaSuccess) return e;
   uint32_t* sched = asched_base();
   if (sched == nullptr) return cudaErrorInvalidSymbol;
   sched += 2 * (seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
-  adamw_requantize_kernel<G><<<static_cast<unsigned>(blocks), kThreads, kSmemBytes, stream>>>(
+  adamw_requantize_kernel<G, kMode><<<static_cast<unsigned>(blocks), kThreads, kSmemBytes, stream>>>(
       a, sched, status);
   return cudaGetLastError();
+}
+
+template <int kMode>
+cudaError_t launch_mode(const AdamwArgs& a, int g, int* status, int num_sms, cudaStream_t stream) {
+  switch (g) {
+    case 32: return launch<32, kMode>(a, status, num_sms, stream);
+    case 64: return launch<64, kMode>(a, status, num_sms, stream);
+    case 128: return launch<128, kMode>(a, status, num_sms, stream);
+    case 256: return launch<256, kMode>(a, status, num_sms, stream);
+    case 512: return launch<512, kMode>(a, status, num_sms, stream);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace
 
 cudaError_t launch_adamw_requantize(const AdamwArgs& a, int g, int* status, int num_sms,
                                     cudaStream_t stream) {
-  switch (g) {
-    case 32: return launch<32>(a, status, num_sms, stream);
-    case 64: return launch<64>(a, status, num_sms, stream);
-    case 128: return launch<128>(a, status, num_sms, stream);
-    case 256: return launch<256>(a, status, num_sms, stream);
-    case 512: return launch<512>(a, status, num_sms, stream);
-    default: return cudaErrorInvalidValue;
-  }
+  if (a.codes == nullptr) return launch<128, kPlain>(a, status, num_sms, stream);
+  return a.given_scale != nullptr ? launch_mode<kGivenScales>(a, g, status, num_sms, stream)
+                                  : launch_mode<kAbsmean>(a, g, status, num_sms, stream);
 }
 
 }  // namespace tq

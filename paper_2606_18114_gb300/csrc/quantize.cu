@@ -60,7 +60,7 @@ __device__ __forceinline__ int find_stage_mat(const QuantMat* mats, int count, i
   return lo;
 }
 
-template <int G, int kMax>
+template <int G, int kMax, bool kGiven>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     quantize_kernel(const __grid_constant__ QuantBatch<kMax> b, uint32_t* sched, int* status) {
   static_assert(G == 32 || G == 64 || G == 128 || G == 256 || G == 512, "group size");
@@ -178,10 +178,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       for (int j = 0; j < 4; ++j) v[j] = src[j];
       const float x[16] = {v[0].x, v[0].y, v[0].z, v[0].w, v[1].x, v[1].y, v[1].z, v[1].w,
                            v[2].x, v[2].y, v[2].z, v[2].w, v[3].x, v[3].y, v[3].z, v[3].w};
-      const bool given = mt.given_scale != nullptr;  // uniform: one matrix per stage
       float s = 0.f;
       uint32_t word;
-      if (given) {
+      if constexpr (kGiven) {
         // the learnable-scale variant: the caller's scale decides, of either sign
         word = code_word_any(x, __ldg(mt.given_scale + e / G), live);
       } else {
@@ -207,7 +206,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
           __reduce_add_sync(gmask, static_cast<unsigned>(16 - __popc(word & 0x55555555u))));
       mt.codes[e >> 4] = word;
       if ((lane & (kLanesPerGroup - 1)) == 0) {
-        if (!given) mt.scales[e / G] = s;
+        if (!kGiven) mt.scales[e / G] = s;
         mt.zeros[e / G] = zc;
       }
     }
@@ -235,32 +234,32 @@ uint32_t* sched_base() {
   return static_cast<uint32_t*>(p);
 }
 
-template <int G, int kMax>
+template <int G, int kMax, bool kGiven>
 cudaError_t launch(const QuantBatch<kMax>& b, int* status, int num_sms, cudaStream_t stream) {
   static std::atomic<uint32_t> seq{0};
   if (b.nstages <= 0) return cudaSuccess;
   if (b.nstages >= (int64_t{1} << 31)) return cudaErrorInvalidValue;
   const int64_t cap = static_cast<int64_t>(num_sms) * kCtasPerSm;
   const int64_t blocks = b.nstages < cap ? b.nstages : cap;
-  cudaError_t e = ensure_smem_limit<quantize_kernel<G, kMax>>(kSmemBytes);
+  cudaError_t e = ensure_smem_limit<quantize_kernel<G, kMax, kGiven>>(kSmemBytes);
   if (e != cudaSuccess) return e;
   uint32_t* sched = sched_base();
   if (sched == nullptr) return cudaErrorInvalidSymbol;
   sched += 2 * (seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
-  quantize_kernel<G, kMax><<<static_cast<unsigned>(blocks), kThreads, kSmemBytes, stream>>>(
+  quantize_kernel<G, kMax, kGiven><<<static_cast<unsigned>(blocks), kThreads, kSmemBytes, stream>>>(
       b, sched, status);
   return cudaGetLastError();
 }
 
-template <int kMax>
+template <int kMax, bool kGiven>
 cudaError_t launch_g(const QuantBatch<kMax>& b, int g, int* status, int num_sms,
                      cudaStream_t stream) {
   switch (g) {
-    case 32: return launch<32, kMax>(b, status, num_sms, stream);
-    case 64: return launch<64, kMax>(b, status, num_sms, stream);
-    case 128: return launch<128, kMax>(b, status, num_sms, stream);
-    case 256: return launch<256, kMax>(b, status, num_sms, stream);
-    case 512: return launch<512, kMax>(b, status, num_sms, stream);
+    case 32: return launch<32, kMax, kGiven>(b, status, num_sms, stream);
+    case 64: return launch<64, kMax, kGiven>(b, status, num_sms, stream);
+    case 128: return launch<128, kMax, kGiven>(b, status, num_sms, stream);
+    case 256: return launch<256, kMax, kGiven>(b, status, num_sms, stream);
+    case 512: return launch<512, kMax, kGiven>(b, status, num_sms, stream);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -484,7 +483,8 @@ cudaError_t launch_quantize(const float* w, int64_t n, int64_t k, int g, uint32_
   b.mats[0] = QuantMat{w, codes, scales, zeros, n * k, 0, row_factor, k, given_scale};
   b.count = 1;
   b.nstages = (n * k + kStageW - 1) / kStageW;
-  return launch_g<1>(b, g, status, num_sms, stream);
+  return given_scale != nullptr ? launch_g<1, true>(b, g, status, num_sms, stream)
+                                 : launch_g<1, false>(b, g, status, num_sms, stream);
 }
 
 cudaError_t launch_quantize_batched(QuantBatch<kQuantMaxMats>& b, int g, int* status,
@@ -495,7 +495,7 @@ cudaError_t launch_quantize_batched(QuantBatch<kQuantMaxMats>& b, int g, int* st
     st += (b.mats[d].total + kStageW - 1) / kStageW;
   }
   b.nstages = st;
-  return launch_g<kQuantMaxMats>(b, g, status, num_sms, stream);
+  return launch_g<kQuantMaxMats, false>(b, g, status, num_sms, stream);
 }
 
 }  // namespace tq
