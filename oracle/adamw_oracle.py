@@ -16,7 +16,7 @@ weight matrix followed by that requantization:
       w  = w * (1 - lr * wd) - (lr / (1 - beta1^t)) * m / (sqrt(v) / sqrt(1 - beta2^t) + eps)
 * then ``tq_oracle.quantize`` of the new w (scales, ternary codes, zero counts).
 
-Readings of points the paper leaves open (also listed in the design doc):
+Readings of points the paper leaves open:
 
 * eps is not given; the default of the common AdamW implementation, 1e-8.
 * The update runs in fp32, the precision of the latent weights, because the new

@@ -16,7 +16,7 @@ threshold to 0.8 x absmean on the gate rows (rows 0..4095 of in_proj). Restated:
 * dalpha_g = sum_{i in group} dW^_i * c_i             (the magnitude's gradient; dW^ = dY^T X,
                                                        the same matrix the STE hands to W)
 
-Readings (also listed in the design doc): the threshold factor multiplies the fp32
+Readings: the threshold factor multiplies the fp32
 absmean in fp32; with f_n = 1 everything reduces to ``tq_oracle.quantize``; the
 magnitude's gradient is the plain chain rule of W^ = alpha * c with c held fixed
 (the codes do not depend on alpha), accumulated in fp64.

@@ -8,7 +8,7 @@ scale of §3.1 with a scale trained as a parameter (``nn.Parameter``), which let
 the zero ratio run away to 90 %. The quantizer is the one of §3.1 with the
 scale taken from the parameter instead of the weights; the paper does not write
 out the gradient that reaches the scale. Restated, with the readings this
-oracle takes (each also listed in the design doc):
+oracle takes:
 
 * c_i  = round(clip(w_i / s_g, -1, 1)), the quotient in fp32 as §3.1's code
          decision, round half to even; for a scale of either sign (a negative

@@ -16,7 +16,7 @@ Module") of the paper, in numpy, in fp64 except where noted:
                                          dX = dY W^
                                          dW = dY^T X         (to the latent W)
 
-Readings of points the paper leaves open (each also listed in the design doc):
+Readings of points the paper leaves open:
 
 * "round" is round-half-to-even (``np.rint``). Only |w/s| = 0.5 is a tie that
   matters (1.5 rounds to 2, which the clip maps to 1 like 1.49 does).
