@@ -30,8 +30,10 @@
 // barriers: a suspended waiter resumed late after an arrival from the other SM.
 //
 // Persistent: the pairs walk the tiles, k-tiles fastest, so that the pairs in
-// flight stream the same dy columns. x is loaded with an L2 evict-last policy (it
-// is re-read by every n-tile and fits in L2), dy with evict-first. Two TMEM
+// flight stream the same dy columns. Both operands are loaded with an L2
+// evict-last policy: x is re-read by every n-tile, and a dy block by the eight
+// pairs of its n-tile, which drift apart in token (with dy evict-first the pair
+// kernel read 1.1 GB from HBM per in_proj launch, and ran 3 % slower). Two TMEM
 // accumulators (2 x 256 columns) let the epilogue of one tile overlap the main loop
 // of the next. Roles: warp 0 TMA, warp 1 MMA (leader) or relay (peer), warps 2-5
 // epilogue; the epilogue thread of lane k writes dW[n][k], so a warp store covers
@@ -44,8 +46,7 @@
 // pieces has each CTA's half of each piece written to the workspace (two slots per
 // CTA: the piece that opens its run and the one that closes it); for each half, the
 // CTA that completes the last piece (a per-tile, per-half counter) adds the pieces
-// in k order and writes dW. No CTA waits for another pair. The tail's pairs read
-// their runs' tokens at different offsets, so there dy is kept in L2 (evict-last).
+// in k order and writes dW. No CTA waits for another pair.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -197,7 +198,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // ---------------------------------------------------------------- TMA producer
     if (lane == 0) {
       const uint64_t keep = policy_evict_last();
-      const uint64_t stream = policy_evict_first();
       int issued = 0;
       bool ok = true;
       for (int i = 0; i < my_items && ok; ++i) {
@@ -219,7 +219,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int c = 0; c < 2; ++c)
             tma_load_2d_hint(b + c * kBox, &tmap_dy, full_bar(s), static_cast<int32_t>(n0 + 64 * c),
-                             mrow, wi.sk < 0 ? stream : keep);
+                             mrow, keep);
           ++issued;
         }
       }
