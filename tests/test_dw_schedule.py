@@ -1,0 +1,102 @@
+"""Host model of the dW kernel's work split (csrc/dw_gemm.cu, CTA pairs with a
+stream-K tail), checked for every schedule shape it can meet: each (tile, k-block) is
+computed exactly once, a split tile's pieces are contiguous and in k order, the
+fixup reads each piece from the workspace slot its writer used, no run needs more
+than its two slots, and every counter and slot index stays inside the device arrays.
+The model restates the scheduler's integer arithmetic; no GPU is involved."""
+import itertools
+
+import pytest
+
+MAX_CTAS = 160  # kDwMaxCtas: workspace of two half-tiles per CTA, a counter per tail half
+
+
+class Sched:
+    def __init__(self, tiles, grid, nkb):
+        self.grid, self.nkb = grid, nkb
+        self.rem = tiles % grid
+        self.units = self.rem * nkb
+        if self.units < grid:
+            self.rem, self.units = 0, 0
+        self.dp = tiles - self.rem
+
+    def run_start(self, c):
+        return c * self.units // self.grid
+
+    def owner(self, b):
+        return ((b + 1) * self.grid - 1) // self.units
+
+    def whole_of(self, c):
+        return (self.dp - 1 - c) // self.grid + 1 if c < self.dp else 0
+
+    def items(self, c):
+        out = [(c + i * self.grid, 0, self.nkb, -1) for i in range(self.whole_of(c))]
+        if self.rem:
+            s0, s1 = self.run_start(c), self.run_start(c + 1)
+            if s1 > s0:
+                for j in range((s1 - 1) // self.nkb - s0 // self.nkb + 1):
+                    r = s0 // self.nkb + j
+                    b0 = r * self.nkb
+                    out.append((self.dp + r, max(s0, b0) - b0, min(s1, b0 + self.nkb) - b0, j))
+        return out
+
+
+def _check(tiles, pairs, nkb):
+    q = Sched(tiles, pairs, nkb)
+    done = {}
+    slot_of = {}  # (pair, tile) -> slot its piece was written to
+    for c in range(pairs):
+        its = q.items(c)
+        nonwhole = [it for it in its if not (it[1] == 0 and it[2] == nkb)]
+        assert len(nonwhole) <= 2, (tiles, pairs, nkb, c, its)
+        for t, kb0, kb1, sk in its:
+            assert 0 <= kb0 < kb1 <= nkb
+            for kb in range(kb0, kb1):
+                assert (t, kb) not in done, ("twice", t, kb)
+                done[(t, kb)] = c
+            if not (kb0 == 0 and kb1 == nkb):
+                assert sk >= 0
+                slot_of[(c, t)] = 0 if sk == 0 else 1
+    assert len(done) == tiles * nkb, "some (tile, k-block) never computed"
+    for r in range(q.rem):
+        t = q.dp + r
+        b0 = r * nkb
+        c_first, c_last = q.owner(b0), q.owner(b0 + nkb - 1)
+        pieces = c_last - c_first + 1
+        for p in range(pieces):  # piece p from pair c_first + p, in k order
+            pc = c_first + p
+            kbs = sorted(kb for (tt, kb), c in done.items() if tt == t and c == pc)
+            assert kbs, (t, p)
+            if pieces > 1:
+                # the slot the fixup reads is the one the writer used
+                assert slot_of[(pc, t)] == (0 if q.run_start(pc) >= b0 else 1)
+            if p > 0:
+                prev = max(kb for (tt, kb), c in done.items() if tt == t and c == pc - 1)
+                assert kbs[0] == prev + 1
+        for rank in (0, 1):
+            assert 2 * r + rank < MAX_CTAS  # completion counter
+    for c in range(pairs):
+        for rank in (0, 1):
+            for j in (0, 1):
+                assert 2 * (2 * c + rank) + j < 2 * MAX_CTAS  # workspace slot
+
+
+@pytest.mark.parametrize("tiles,pairs,nkb", [
+    (272, 76, 256),   # Mamba-2 in_proj: 34 x 8 pair tiles, 16384 tokens
+    (128, 76, 256),   # out_proj: 8 x 16 pair tiles
+    (76, 76, 256),    # exactly one wave
+    (77, 76, 1),      # a tail with fewer k-blocks than pairs: whole tiles
+    (3, 2, 5),
+    (1, 1, 1),
+    (1, 1, 2048),     # one tile, one pair: 131072 tokens
+])
+def test_dw_pair_schedule_shapes(tiles, pairs, nkb):
+    _check(tiles, pairs, nkb)
+
+
+def test_dw_pair_schedule_sweep():
+    for tiles, pairs, nkb in itertools.product([1, 2, 5, 37, 75, 76, 77, 151, 152, 272],
+                                               [1, 2, 3, 38, 75, 76, 80],
+                                               [1, 2, 3, 7, 16, 64, 257]):
+        if pairs <= tiles:
+            _check(tiles, pairs, nkb)
