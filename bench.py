@@ -737,7 +737,13 @@ def run_only(args):
     p = Prefill(tq, IN_PROJ[0], IN_PROJ[1], M_PREFILL, G, seed=7)
     tq.quantize(p.w, p.g, out=(p.codes, p.s, p.z))
     tq.codes_transpose(p.codes, p.k, out=p.codes_t)
+    dwr = torch.randn((p.n, p.k), device="cuda") * 1e-3
+    sg = p.s * 1.1  # given scales of the learnable-scale variant
+    ds, da = torch.empty_like(p.s), torch.empty_like(p.s)
     calls.update({
+        "given": lambda: tq.quantize_with_scales(p.w, p.g, sg, out=(p.codes, p.z)),
+        "scale_grad": lambda: tq.scale_grad(p.w, dwr, p.codes, sg, p.g, out=ds),
+        "alpha_grad": lambda: tq.alpha_grad(dwr, p.codes, p.g, out=da),
         "quantize": lambda: tq.quantize(p.w, p.g, out=(p.codes, p.s, p.z)),
         "transpose": lambda: tq.codes_transpose(p.codes, p.k, out=p.codes_t),
         "fwd": lambda: tq.linear_fwd(p.x, p.codes, p.s, p.g, y=p.y),
@@ -770,7 +776,8 @@ def main():
     ap.add_argument("--impl", default="tq", choices=["tq", "reference"])
     ap.add_argument("--no-extra", action="store_true", help="skip decode/quantize sweeps")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
-    ap.add_argument("--only", choices=["quantize", "transpose", "fwd", "dx", "dw", "decode", "adamw"],
+    ap.add_argument("--only", choices=["quantize", "transpose", "fwd", "dx", "dw", "decode", "adamw",
+                                       "given", "scale_grad", "alpha_grad"],
                     help="profiling aid: run just this kernel of the step (or the batched "
                          "M=1 decode) --warmup + --steps times and print its time")
     args = ap.parse_args()
