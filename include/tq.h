@@ -269,6 +269,9 @@ TQ_API tq_status tq_linear_fwd(const void* x, int64_t m, int64_t k,
  *                dX expands the codes of W^T like the forward expands W's (faster);
  *                NULL makes dX read `codes` directly.
  *   Requires k % 64 == 0, k % g == 0, n % 8 == 0. x may be NULL when dw is.
+ *   dW launches of one device share a library workspace (the partial sums of the
+ *   tiles split across SMs): a dW issued on another stream than the previous one
+ *   is ordered after it by the library (an event wait on the new stream).
  */
 TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t n, int64_t k,
                         const uint32_t* codes, const uint32_t* codes_t, const float* scales,
