@@ -435,6 +435,13 @@ int resident_pairs(int num_sms) {
 
 size_t dw_smem_bytes() { return kBytes + 1024; }
 
+cudaError_t reset_dw_counters() {
+  void* p = nullptr;
+  cudaError_t e = cudaGetSymbolAddress(&p, g_dw_cnt);
+  if (e != cudaSuccess) return e;
+  return cudaMemset(p, 0, sizeof(g_dw_cnt));
+}
+
 cudaError_t launch_dw_gemm(const CUtensorMap& tmap_x, const CUtensorMap& tmap_dy,
                            const DwArgs& a, int num_sms, cudaStream_t stream) {
   const size_t smem = dw_smem_bytes();

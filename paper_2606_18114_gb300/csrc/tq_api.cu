@@ -316,6 +316,12 @@ tq_status check_fwd_args(const void* x, int64_t m, int64_t k, const uint32_t* co
 
 }  // namespace
 
+namespace tq {
+// dw_gemm.cu: zero the stream-K completion counters (after a launch gave up on a
+// wait, when the CTA that would have reset them may not have run). Synchronous.
+cudaError_t reset_dw_counters();
+}  // namespace tq
+
 extern "C" {
 
 TQ_API const char* tq_last_error(void) { return g_err; }
@@ -722,6 +728,8 @@ TQ_API tq_status tq_device_status(void* stream) {
     const int zero = 0;
     if ((e = cudaMemcpy(dev->status, &zero, sizeof(int), cudaMemcpyHostToDevice)) != cudaSuccess)
       return cuda_fail(e, "status clear");
+    // a dW launch that gave up may have left tile counters of its stream-K tail set
+    if ((e = tq::reset_dw_counters()) != cudaSuccess) return cuda_fail(e, "dW counter reset");
     return fail(TQ_ERR_TIMEOUT, "a kernel wait ran out (device status %d)", v);
   }
   return TQ_OK;
