@@ -78,27 +78,104 @@ def recorded_traffic(kernel, files):
 
 
 class ClockSampler:
-    """nvidia-smi clock / throttle-reason samples while the timed region runs."""
+    """SM clock, power and clock-event reasons while the timed region runs.
+
+    Polls NVML (the driver's libnvidia-ml, through ctypes) every ~2 ms from a
+    thread; ``mark(True)`` / ``mark(False)`` bracket the timed region on the host
+    (the launches are queued inside it and the final synchronise returns when the
+    device is done), and only samples taken inside the bracket are reported.
+    Falls back to ``nvidia-smi -lms 20`` when NVML cannot be loaded."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    # clock-event reason bits of NVML
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
 
-    def __init__(self, gpu_index: int):
+    def __init__(self, gpu_index: int, period_s: float = 0.002):
         self.idx = gpu_index
+        self.period = period_s
         self.proc = None
+        self.thread = None
+        self.samples = []      # (t, sm_mhz, power_w, reasons bitmask)
+        self.window = [None, None]
+        self.sm_max = None
+        self.source = None
+
+    def _nvml_handle(self):
+        import ctypes
+        lib = None
+        for name in ("libnvidia-ml.so.1", "libnvidia-ml.so"):
+            try:
+                lib = ctypes.CDLL(name)
+                break
+            except OSError:
+                continue
+        if lib is None or lib.nvmlInit_v2() != 0:
+            return None, None
+        h = ctypes.c_void_p()
+        uuid = None
+        try:
+            uuid = str(torch.cuda.get_device_properties(self.idx).uuid)
+        except Exception:
+            pass
+        ok = False
+        if uuid:
+            for u in (uuid, "GPU-" + uuid):
+                if lib.nvmlDeviceGetHandleByUUID(u.encode(), ctypes.byref(h)) == 0:
+                    ok = True
+                    break
+        if not ok and lib.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(self.idx), ctypes.byref(h)) != 0:
+            return None, None
+        return lib, h
+
+    def _poll(self, lib, h):
+        import ctypes
+        clk, pw, mx = ctypes.c_uint(), ctypes.c_uint(), ctypes.c_uint()
+        rs = ctypes.c_ulonglong()
+        get_reasons = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            getattr(lib, "nvmlDeviceGetCurrentClocksThrottleReasons")
+        if lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:
+            self.sm_max = float(mx.value)
+        while not self._stop:
+            t = time.perf_counter()
+            if lib.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0:
+                p = pw.value / 1000.0 if lib.nvmlDeviceGetPowerUsage(h, ctypes.byref(pw)) == 0 else None
+                r = rs.value if get_reasons(h, ctypes.byref(rs)) == 0 else 0
+                self.samples.append((t, float(clk.value), p, int(r)))
+            time.sleep(self.period)
+
+    def mark(self, start: bool):
+        self.window[0 if start else 1] = time.perf_counter()
 
     def __enter__(self):
+        import threading
+        self._stop = False
+        lib, h = (None, None)
+        try:
+            lib, h = self._nvml_handle()
+        except Exception:
+            lib = None
+        if lib is not None:
+            self.source = "nvml, 2 ms"
+            self.thread = threading.Thread(target=self._poll, args=(lib, h), daemon=True)
+            self.thread.start()
+            return self
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.source = "nvidia-smi, 20 ms"
         except (OSError, ValueError):
             self.proc = None
         return self
 
     def __exit__(self, *exc):
+        self._stop = True
+        if self.thread is not None:
+            self.thread.join(timeout=5)
         self.out = ""
         if self.proc is not None:
             self.proc.terminate()
@@ -109,6 +186,19 @@ class ClockSampler:
                 self.out, _ = self.proc.communicate()
 
     def summary(self):
+        if self.thread is not None:
+            t0, t1 = self.window
+            inside = [s for s in self.samples
+                      if (t0 is None or s[0] >= t0) and (t1 is None or s[0] <= t1)]
+            if not inside:
+                return {"sm_mhz": None, "sm_max_mhz": self.sm_max, "reasons": ["no sample"],
+                        "samples": 0, "source": self.source}
+            names = sorted({nm for s in inside for bit, nm in self.REASONS.items() if s[3] & bit})
+            pw = [s[2] for s in inside if s[2] is not None]
+            return {"sm_mhz": statistics.median(s[1] for s in inside), "sm_max_mhz": self.sm_max,
+                    "sm_mhz_min": min(s[1] for s in inside), "reasons": names,
+                    "samples": len(inside), "power_w_max": max(pw) if pw else None,
+                    "source": self.source}
         rows = [r for r in csv.reader(io.StringIO(self.out or "")) if len(r) >= 9]
         if not rows:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
@@ -120,7 +210,7 @@ class ClockSampler:
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(smax) if smax else None,
                 "reasons": reasons, "samples": len(rows),
-                "power_w_max": max(pw) if pw else None}
+                "power_w_max": max(pw) if pw else None, "source": self.source}
 
 
 def dist_setup(n_gpus, backend=None):
@@ -221,7 +311,7 @@ KERNELS = [  # name, source files, event span
 ]
 
 
-def time_prefill(p: Prefill, steps, warmup, world):
+def time_prefill(p: Prefill, steps, warmup, world, clk=None):
     for _ in range(warmup):
         p.step()
     torch.cuda.synchronize()
@@ -230,11 +320,15 @@ def time_prefill(p: Prefill, steps, warmup, world):
     torch.cuda.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
+    if clk is not None:
+        clk.mark(True)
     t0.record()
     for i in range(steps):
         p.step(evs[i])
     t1.record()
     torch.cuda.synchronize()
+    if clk is not None:
+        clk.mark(False)
     barrier(world)
     total_ms = t0.elapsed_time(t1)
     per = {}
@@ -797,13 +891,22 @@ def main():
     rank, world, local = dist_setup(args.gpus)
     p = Prefill(tq, IN_PROJ[0], IN_PROJ[1], M_PREFILL, G, seed=1000 + rank)
     with ClockSampler(local) as clk:
-        total_ms, per = time_prefill(p, args.steps, args.warmup, world)
+        total_ms, per = time_prefill(p, args.steps, args.warmup, world, clk)
     total_ms = max_over_ranks(total_ms, world)
     rate, ms = whole_job(p.flops, world, total_ms, args.steps)
     value = rate / 1e12
 
     pk, pk_kind = peaks()
     gemm_flops = 2.0 * p.m * p.n * p.k
+    # The measured peaks are a burst (best of 10 GEMMs) and a sustained figure (4 s of
+    # back-to-back GEMMs at the power cap): a timed region of under a second takes
+    # the burst peak, a longer one the sustained peak.
+    region_s = total_ms / 1e3
+    sustained = region_s >= 1.0
+    tc_peak = pk["bf16_tflops_sustained"] if sustained else pk["bf16_tflops"]
+    peak_rule = (f"{pk_kind} bf16 dense {'sustained' if sustained else 'burst'}: the timed region "
+                 f"({args.steps} steps) lasted {region_s * 1e3:.1f} ms, "
+                 f"{'at least' if sustained else 'under'} 1 s")
     kinfo = {}
     for name, files, _ in KERNELS:
         t = per[name]
@@ -813,21 +916,23 @@ def main():
             kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "GB/s",
                            "frac": round(ach / pk["hbm_gbs"], 4)}
         else:
-            # timed inside the long step loop, at the power cap: the sustained peak
-            # is the denominator; the burst fraction is kept beside it
             ach = gemm_flops / (t * 1e-3) / 1e12
             kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "TFLOP/s",
-                           "frac": round(ach / pk["bf16_tflops_sustained"], 4),
-                           "frac_of_burst": round(ach / pk["bf16_tflops"], 4)}
+                           "frac": round(ach / tc_peak, 4),
+                           "frac_of_burst": round(ach / pk["bf16_tflops"], 4),
+                           "frac_of_sustained": round(ach / pk["bf16_tflops_sustained"], 4)}
     dom = max((n for n, _, _ in KERNELS if n not in ("quantize", "transpose")), key=lambda n: per[n])
     dom_files = dict((n, f) for n, f, _ in KERNELS)[dom]
     roof = {"kernel": dom, "bound": "tensor", "achieved": kinfo[dom]["achieved"],
-            "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s", "frac": kinfo[dom]["frac"],
+            "peak": tc_peak, "unit": "TFLOP/s", "frac": kinfo[dom]["frac"],
             "traffic": recorded_traffic(dom, dom_files),
-            "peak_kind": f"{pk_kind} bf16 dense, sustained (the kernel is timed inside the "
-                         f"{args.steps}-step loop, at the power cap)",
+            "peak_kind": peak_rule, "timed_region_ms": round(total_ms, 3),
             "frac_of_burst": kinfo[dom]["frac_of_burst"], "burst_peak": pk["bf16_tflops"],
-            "algorithmic_per_launch": gemm_flops}
+            "frac_of_sustained": kinfo[dom]["frac_of_sustained"],
+            "sustained_peak": pk["bf16_tflops_sustained"],
+            "algorithmic_per_launch": gemm_flops,
+            "achieved_how": "algorithmic flops per launch / mean CUDA-event time of the "
+                            "kernel's launch inside the timed steps"}
 
     e2e_steps = max(5, args.steps // 10)
     barrier(world)

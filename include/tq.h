@@ -14,7 +14,11 @@
  *     16-byte aligned. The library keeps no pointer after a call returns.
  *   - Work is enqueued on `stream` (a cudaStream_t passed as void*; NULL is the
  *     legacy default stream). No entry point synchronises, except
- *     tq_device_status(). No entry point allocates device memory.
+ *     tq_device_status(). No entry point allocates device memory. The library
+ *     holds fixed file-scope device arrays instead, present on every device
+ *     that loads it until the process exits: 40 MB of dW stream-K workspace
+ *     (tq_linear_bwd), 16 MB of transposed-code scratch (tq_linear_bwd_noalloc),
+ *     and a few KB of work counters and status words.
  *   - Arguments are checked before anything is enqueued. A rejected call
  *     returns TQ_ERR_INVALID_ARG or TQ_ERR_UNSUPPORTED, writes nothing and
  *     leaves a message in tq_last_error().
@@ -269,9 +273,10 @@ TQ_API tq_status tq_linear_fwd(const void* x, int64_t m, int64_t k,
  *                dX expands the codes of W^T like the forward expands W's (faster);
  *                NULL makes dX read `codes` directly.
  *   Requires k % 64 == 0, k % g == 0, n % 8 == 0. x may be NULL when dw is.
- *   dW launches of one device share a library workspace (the partial sums of the
- *   tiles split across SMs): a dW issued on another stream than the previous one
- *   is ordered after it by the library (an event wait on the new stream).
+ *   dW launches of one device share the library's 40 MB workspace (the partial
+ *   sums of the tiles split across SMs): each dW launch waits for the device's
+ *   previous dW launch, on whatever stream either was issued (an event the
+ *   library records after every dW launch, waited on by the next one).
  */
 TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t n, int64_t k,
                         const uint32_t* codes, const uint32_t* codes_t, const float* scales,
@@ -334,6 +339,9 @@ TQ_API tq_status tq_linear_fwd_batched(const tq_fwd_desc* descs, int32_t count, 
  * tq_device_status — synchronises `stream`, then returns and clears the status
  * word of the current device: TQ_OK, or TQ_ERR_TIMEOUT if a kernel's bounded
  * wait ran out since the last call; TQ_ERR_CUDA if the synchronise failed.
+ * On TQ_ERR_TIMEOUT it first synchronises the whole device (every stream), then
+ * clears the word and zeroes the dW kernel's stream-K tile counters, which a
+ * launch that gave up may have left set; later calls then run normally.
  */
 TQ_API tq_status tq_device_status(void* stream);
 

@@ -435,6 +435,13 @@ int resident_pairs(int num_sms) {
 
 size_t dw_smem_bytes() { return kBytes + 1024; }
 
+// Order of the device's dW launches (they share the workspace above): the event
+// of the last launch, and whether there was one.
+constexpr int kOrderDevices = 64;
+static std::mutex g_dw_order_mu;
+static cudaEvent_t g_dw_done[kOrderDevices] = {};
+static bool g_dw_launched[kOrderDevices] = {};
+
 cudaError_t reset_dw_counters() {
   void* p = nullptr;
   cudaError_t e = cudaGetSymbolAddress(&p, g_dw_cnt);
@@ -453,27 +460,22 @@ cudaError_t launch_dw_gemm(const CUtensorMap& tmap_x, const CUtensorMap& tmap_dy
   if (pairs > kDwMaxCtas / 2) pairs = kDwMaxCtas / 2;
   if (pairs < 1) pairs = 1;
   // The stream-K workspace and counters are shared by the device's dW launches:
-  // a launch on another stream than the previous one waits for it.
-  static std::mutex mu;
-  static cudaEvent_t done[64] = {};
-  static cudaStream_t last[64] = {};
+  // every launch after the first waits for the previous one, whatever stream
+  // either was issued on (a wait on the same stream's own last event costs
+  // nothing on the device).
+  std::lock_guard<std::mutex> lock(g_dw_order_mu);
   int dev = 0;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-  std::lock_guard<std::mutex> lock(mu);
-  if (dev < 64) {
-    if (done[dev] == nullptr &&
-        (e = cudaEventCreateWithFlags(&done[dev], cudaEventDisableTiming)) != cudaSuccess)
-      return e;
-    if (last[dev] != stream && last[dev] != nullptr &&
-        (e = cudaStreamWaitEvent(stream, done[dev], 0)) != cudaSuccess)
-      return e;
-  }
+  if (dev >= kOrderDevices) return cudaErrorInvalidDevice;
+  if (g_dw_done[dev] == nullptr &&
+      (e = cudaEventCreateWithFlags(&g_dw_done[dev], cudaEventDisableTiming)) != cudaSuccess)
+    return e;
+  if (g_dw_launched[dev] && (e = cudaStreamWaitEvent(stream, g_dw_done[dev], 0)) != cudaSuccess)
+    return e;
   dw_gemm_kernel<<<static_cast<unsigned>(2 * pairs), kThreads, smem, stream>>>(tmap_x, tmap_dy, a);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  if (dev < 64) {
-    if ((e = cudaEventRecord(done[dev], stream)) != cudaSuccess) return e;
-    last[dev] = stream;
-  }
+  if ((e = cudaEventRecord(g_dw_done[dev], stream)) != cudaSuccess) return e;
+  g_dw_launched[dev] = true;
   return cudaSuccess;
 }
 

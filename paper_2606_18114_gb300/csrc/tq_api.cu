@@ -725,6 +725,9 @@ TQ_API tq_status tq_device_status(void* stream) {
   if ((e = cudaMemcpy(&v, dev->status, sizeof(int), cudaMemcpyDeviceToHost)) != cudaSuccess)
     return cuda_fail(e, "status read");
   if (v != 0) {
+    // Work of every stream of the device ends before the reset: a dW launch still
+    // running on another stream would otherwise race with it.
+    if ((e = cudaDeviceSynchronize()) != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
     const int zero = 0;
     if ((e = cudaMemcpy(dev->status, &zero, sizeof(int), cudaMemcpyHostToDevice)) != cudaSuccess)
       return cuda_fail(e, "status clear");
@@ -780,6 +783,10 @@ TQ_API tq_status tq_linear_bwd_noalloc(const void* dy, const void* x, int64_t m,
                 "transposed codes of n=%lld k=%lld need %lld words, scratch holds %lld; pass "
                 "codes_t to tq_linear_bwd instead",
                 (long long)n, (long long)k, (long long)(ldt * k), (long long)kNoAllocWords);
+  // the device and architecture check before the scratch's address is looked up
+  // (an unsupported device gets TQ_ERR_UNSUPPORTED, as from every entry point)
+  const DeviceInfo* devinfo = nullptr;
+  TQ_TRY(device_info(&devinfo));
   uint32_t* scratch = nullptr;
   TQ_TRY(noalloc_scratch(&scratch));
   const cudaError_t e =
