@@ -345,6 +345,24 @@ TQ_API tq_status tq_linear_fwd_batched(const tq_fwd_desc* descs, int32_t count, 
  */
 TQ_API tq_status tq_device_status(void* stream);
 
+/*
+ * tq_test_hooks — for testing the timeout path only; the paper has no counterpart.
+ * Sets, for every later launch on the current device, the time limit of every
+ * kernel wait (wait_limit_ns > 0; 0 restores the default of 2 s) and test flags
+ * that make one kernel role withhold its first arrival on a barrier (0 in normal
+ * use):
+ *   1  tq_quantize / tq_quantize_batched: consumer warp 0 of CTA 0 does not
+ *      release its first stage, so the producer's wait for that slot runs out;
+ *   2  the dW product of tq_linear_bwd: the first epilogue warp of the first CTA
+ *      pair's leader does not release its first accumulator, so the MMA issuer's
+ *      wait for it runs out.
+ * A launch made while a flag is set winds down at the limit (no copy or MMA left
+ * in flight, every wait bounded) and reports TQ_ERR_TIMEOUT through
+ * tq_device_status(); its outputs are undefined. Synchronises the device first.
+ * Returns TQ_ERR_INVALID_ARG for a negative limit or an unknown flag.
+ */
+TQ_API tq_status tq_test_hooks(int64_t wait_limit_ns, uint32_t flags);
+
 /* Message of the last failure on the calling thread ("" if none). */
 TQ_API const char* tq_last_error(void);
 

@@ -4,7 +4,8 @@
 // bytes per weight at g = 128).
 //
 // Work unit = a block of 256 consecutive weight rows of one matrix over its
-// whole K. Per CTA (one per SM) a producer warp claims units one at a time from
+// whole K. Per CTA (one per SM) a producer warp takes unit blockIdx.x first (no
+// claim latency before the first load), then claims units one at a time from
 // a per-launch global counter, in order, with the matrices of the batch sorted
 // by decreasing K (the last units claimed are the shortest; SMs do not all
 // receive HBM data at the same rate, so static shares leave SMs idle). It
@@ -153,18 +154,19 @@ __device__ __forceinline__ uint32_t opaque(uint32_t v) {
   return r;
 }
 
-// mma.sync m16n8k16, A and B in the activation type (both bf16, or both fp16).
+// mma.sync m16n8k16, A and B in the activation type (both bf16, or both fp16). Not
+// volatile: the compiler may interleave the independent chains of a warp.
 template <bool F16>
 __device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                          uint32_t a3, uint32_t b0, uint32_t b1) {
   if constexpr (F16)
-    asm volatile(
+    asm(
         "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, "
         "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
   else
-    asm volatile(
+    asm(
         "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
         "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
@@ -176,13 +178,13 @@ template <bool F16>
 __device__ __forceinline__ void mma16816_zc(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                             uint32_t a3, uint32_t b0, uint32_t b1) {
   if constexpr (F16)
-    asm volatile(
+    asm(
         "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, "
         "{%4, %5, %6, %7}, {%8, %9}, {%10, %10, %10, %10};"
         : "=f"(c[0]), "=f"(c[1]), "=f"(c[2]), "=f"(c[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(0.0f));
   else
-    asm volatile(
+    asm(
         "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
         "{%4, %5, %6, %7}, {%8, %9}, {%10, %10, %10, %10};"
         : "=f"(c[0]), "=f"(c[1]), "=f"(c[2]), "=f"(c[3])
@@ -291,10 +293,14 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     int64_t issued = 0;
     int units_u = 0;  // units whose scales went through the unit buffers
     bool ok = true;
+    int claims = 0;
     for (;;) {
-      int u = 0;
-      if (lane == 0) u = static_cast<int>(atomicAdd(&sched[0], 1u));
-      u = __shfl_sync(0xffffffffu, u, 0);
+      // the first unit of every CTA is dealt (blocks <= units), later ones claimed
+      int u = static_cast<int>(blockIdx.x);
+      if (claims++ > 0) {
+        if (lane == 0) u = static_cast<int>(gridDim.x + atomicAdd(&sched[0], 1u));
+        u = __shfl_sync(0xffffffffu, u, 0);
+      }
       if (u >= b.total_units) break;
       const int d = find_mat(b, u);
       const DecodeMat& mt = b.mats[d];

@@ -282,10 +282,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     const int row = quad * 32 + lane;  // this thread's TMEM lane: feature k0 + row
     const uint32_t leader_accempty0 = map_to_rank(accempty_bar(0), 0);
+    // timeout tests only: the leader's first epilogue warp of pair 0 withholds its
+    // first "accumulator empty" arrival
+    bool withhold = pair == 0 && rank == 0 && warp == 2 && test_withhold(status, kWithholdDwAccEmpty);
     auto release = [&](int acc) {  // this warp is done with the accumulator
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive_remote(leader_accempty0 + 8u * acc);
+      if (lane == 0 && !withhold) mbar_arrive_remote(leader_accempty0 + 8u * acc);
+      withhold = false;
     };
     // workspace slot of piece j of the run of pair c (its first piece or its last),
     // for this CTA's half

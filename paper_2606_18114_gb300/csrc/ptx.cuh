@@ -1,9 +1,14 @@
 // ptx.cuh — inline-PTX wrappers for sm_103a: mbarrier, TMA, tcgen05 (UMMA + TMEM).
 //
-// Every wait here is bounded: a wait that does not complete within
-// kWaitLimitNs of %globaltimer (or kWaitMaxPolls polls) records TQ_ERR_TIMEOUT
-// in the caller's status word and returns false, so that the kernel can wind
-// down instead of hanging the GPU.
+// Every wait here is bounded: a wait that does not complete within the time
+// limit of %globaltimer (or kWaitMaxPolls polls) records TQ_ERR_TIMEOUT in the
+// caller's status word and returns false, so that the kernel can wind down
+// instead of hanging the GPU.
+//
+// The status word is the first of four words of per-device control state
+// (DeviceCtl): the status, test flags that make one role withhold one arrival
+// (the timeout tests; zero in normal use), and a 64-bit wait limit in ns (zero:
+// kWaitLimitNs). The limit is read only once a wait has not completed at once.
 #pragma once
 
 #include <cuda.h>
@@ -15,6 +20,19 @@ namespace tq {
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 constexpr uint32_t kWaitMaxPolls = 1u << 30;
 constexpr int kStatusTimeout = 4;                 // TQ_ERR_TIMEOUT
+
+// Test flags of DeviceCtl word 1: the role named withholds its first arrival.
+constexpr int kWithholdQuantizeEmpty = 1;  // quantize: consumer warp 0 of CTA 0, "empty"
+constexpr int kWithholdDwAccEmpty = 2;     // dW: leader epilogue warp 2 of pair 0, "acc empty"
+
+__device__ __forceinline__ uint64_t wait_limit_ns(const int* status) {
+  const uint64_t v = *reinterpret_cast<const volatile unsigned long long*>(status + 2);
+  return v != 0 ? v : kWaitLimitNs;
+}
+
+__device__ __forceinline__ bool test_withhold(const int* status, int flag) {
+  return (*reinterpret_cast<const volatile int*>(status + 1) & flag) != 0;
+}
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -87,9 +105,10 @@ __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* status) {
   if (mbar_test_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
+  const uint64_t limit = wait_limit_ns(status);
   for (uint32_t n = 1; n < kWaitMaxPolls; ++n) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (globaltimer_ns() - t0 > kWaitLimitNs) break;
+    if (globaltimer_ns() - t0 > limit) break;
   }
   atomicExch(status, kStatusTimeout);
   return false;
@@ -102,9 +121,10 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* st
 __device__ __forceinline__ bool mbar_wait_spin(uint32_t bar, uint32_t parity, int* status) {
   if (mbar_test_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
+  const uint64_t limit = wait_limit_ns(status);
   for (uint32_t n = 1;; ++n) {
     if (mbar_test_wait(bar, parity)) return true;
-    if ((n & 1023u) == 0 && (globaltimer_ns() - t0 > kWaitLimitNs || n >= kWaitMaxPolls)) break;
+    if ((n & 1023u) == 0 && (globaltimer_ns() - t0 > limit || n >= kWaitMaxPolls)) break;
   }
   atomicExch(status, kStatusTimeout);
   return false;

@@ -159,6 +159,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   // -------------------------------------------------------------- consumers
   int slot = 0;
   uint32_t parity = 0;
+  // timeout tests only: this warp withholds its first "empty" arrival
+  bool withhold = blockIdx.x == 0 && warp == 0 && test_withhold(status, kWithholdQuantizeEmpty);
   for (;;) {
     if (!lanes_wait(full_bar(slot), parity, status)) return;
     const int64_t ls = stage_of[slot];
@@ -211,7 +213,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       }
     }
     __syncwarp();
-    if (lane == 0) mbar_arrive(empty_bar(slot));
+    if (lane == 0 && !withhold) mbar_arrive(empty_bar(slot));
+    withhold = false;
     if (++slot == kStages) {
       slot = 0;
       parity ^= 1u;

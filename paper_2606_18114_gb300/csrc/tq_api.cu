@@ -35,8 +35,11 @@ tq_status cuda_fail(cudaError_t e, const char* what) {
   return fail(TQ_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
 }
 
-// Status word written by kernels whose bounded waits run out (one per device).
-__device__ int g_device_status;
+// Per-device control words passed to every kernel (one set per device): [0] the
+// status word written by kernels whose bounded waits run out, [1] test flags that
+// make one role withhold one arrival (tq_test_hooks; 0 in normal use), [2..3] the
+// wait limit in ns as a 64-bit value (0: the kernels' default).
+__device__ __align__(16) int g_device_ctl[4];
 
 struct DeviceInfo {
   bool ready = false;
@@ -65,7 +68,7 @@ tq_status device_info(const DeviceInfo** out) {
       return fail(TQ_ERR_UNSUPPORTED, "libtq is built for sm_103a (GB300); device %d is sm_%d%d",
                   dev, major, minor);
     void* p = nullptr;
-    if ((e = cudaGetSymbolAddress(&p, g_device_status)) != cudaSuccess)
+    if ((e = cudaGetSymbolAddress(&p, g_device_ctl)) != cudaSuccess)
       return cuda_fail(e, "cudaGetSymbolAddress");
     d.num_sms = sms;
     d.status = static_cast<int*>(p);
@@ -735,6 +738,23 @@ TQ_API tq_status tq_device_status(void* stream) {
     if ((e = tq::reset_dw_counters()) != cudaSuccess) return cuda_fail(e, "dW counter reset");
     return fail(TQ_ERR_TIMEOUT, "a kernel wait ran out (device status %d)", v);
   }
+  return TQ_OK;
+}
+
+TQ_API tq_status tq_test_hooks(int64_t wait_limit_ns, uint32_t flags) {
+  g_err[0] = 0;
+  if (wait_limit_ns < 0) return fail(TQ_ERR_INVALID_ARG, "negative wait limit");
+  if ((flags & ~3u) != 0) return fail(TQ_ERR_INVALID_ARG, "unknown test flags 0x%x", flags);
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaError_t e = cudaDeviceSynchronize();  // no kernel may be reading the words
+  if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
+  int words[3];
+  words[0] = static_cast<int>(flags);
+  const uint64_t lim = static_cast<uint64_t>(wait_limit_ns);
+  memcpy(&words[1], &lim, sizeof(lim));
+  if ((e = cudaMemcpy(dev->status + 1, words, sizeof(words), cudaMemcpyHostToDevice)) != cudaSuccess)
+    return cuda_fail(e, "test hooks write");
   return TQ_OK;
 }
 

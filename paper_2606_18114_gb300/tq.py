@@ -32,6 +32,7 @@ __all__ = [
     "scale_grad",
     "adamw_requantize_with_scales",
     "adamw",
+    "test_hooks",
     "AdamwHparams",
     "version",
     "OUT_F32",
@@ -49,7 +50,7 @@ EXPORTS = ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd
            "tq_linear_bwd_noalloc", "tq_codes_transpose", "tq_linear_fwd_batched",
            "tq_adamw_requantize", "tq_quantize_decoupled", "tq_alpha_grad",
            "tq_quantize_with_scales", "tq_scale_grad", "tq_adamw_requantize_with_scales",
-           "tq_adamw", "tq_device_status", "tq_last_error", "tq_version")
+           "tq_adamw", "tq_device_status", "tq_test_hooks", "tq_last_error", "tq_version")
 
 _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtq.so")
 _lib = None
@@ -126,9 +127,10 @@ def load(path: Optional[str] = None):
     lib.tq_adamw_requantize_with_scales.argtypes = [vp, vp, vp, vp, i64, i64, i32,
                                                     ctypes.POINTER(AdamwHparams), vp, vp, vp, vp]
     lib.tq_adamw.argtypes = [vp, vp, vp, vp, i64, ctypes.POINTER(AdamwHparams), vp]
+    lib.tq_test_hooks.argtypes = [i64, ctypes.c_uint32]
     for name in ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
                  "tq_linear_bwd_noalloc", "tq_codes_transpose", "tq_linear_fwd_batched",
-                 "tq_device_status"):
+                 "tq_device_status", "tq_test_hooks"):
         getattr(lib, name).restype = ctypes.c_int
     lib.tq_last_error.restype = ctypes.c_char_p
     lib.tq_last_error.argtypes = []
@@ -164,6 +166,12 @@ def version() -> str:
 def device_status(stream=None) -> None:
     """Synchronise the stream and raise if a kernel's bounded wait ran out."""
     _check(load().tq_device_status(_stream(stream)))
+
+
+def test_hooks(wait_limit_ns: int = 0, flags: int = 0) -> None:
+    """Timeout-path testing only (include/tq.h, tq_test_hooks): the kernels' wait
+    limit on this device (0: the default) and the withhold-one-arrival flags."""
+    _check(load().tq_test_hooks(int(wait_limit_ns), int(flags)))
 
 
 def quantize(w: torch.Tensor, g: int, out=None, stream=None):

@@ -233,3 +233,10 @@ def test_activation_flag_checked(lib):
     arr[1] = FwdDesc(FAKE, FAKE, FAKE, FAKE, 64, 256, 128, 0x100)
     assert lib.tq_linear_fwd_batched(arr, 2, 4, None) == 1
     assert b"activation type" in lib.tq_last_error()
+
+
+def test_test_hooks_reject_before_device(lib):
+    # argument errors come before any device access
+    assert lib.tq_test_hooks(-1, 0) == 1
+    assert lib.tq_test_hooks(1000, 4) == 1
+    assert b"flags" in lib.tq_last_error()

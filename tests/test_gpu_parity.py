@@ -290,6 +290,49 @@ def test_decode_parity(tq, g, m):
     assert torch.equal(yb, y.to(torch.bfloat16))
 
 
+@pytest.mark.parametrize("m", [1, 2, 3, 4, 6, 7])
+@pytest.mark.parametrize("g", [128, 256, 512])
+def test_decode_activation_ranges(tq, m, g):
+    """Few-token forward with activations over most of the bf16 range: every token
+    scaled by its own power of two from 2^-100 to 2^100, one 128-wide chunk all
+    zero, one chunk spanning 2^-30 .. 2^8 inside itself; each token compared on its
+    own (the oracle's output of that token alone), so that a small token is not
+    hidden by a large one."""
+    n, k = 264, 1536
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=700 + m + g)
+    rs = np.random.default_rng(m * 1000 + g)
+    xf = x.float().numpy().copy()
+    for tok in range(m):
+        e = rs.integers(-100, 101)
+        xf[tok] *= np.float32(2.0 ** float(e))
+    xf[0, 128:256] = 0.0                                         # a zero chunk
+    xf[m - 1, 256:384] = (rs.choice([-1, 1], 128) *
+                          2.0 ** rs.uniform(-30, 8, 128)).astype(np.float32)
+    xb = torch.from_numpy(xf).to(torch.bfloat16)
+    y = tq.linear_fwd(xb.cuda(), codes, s, g)
+    tq.device_status()
+    ref = O.linear_fwd(xb, w_hat)
+    for tok in range(m):
+        check_close(to_np(y[tok:tok + 1]), ref[tok:tok + 1], f"Y token {tok} m={m} g={g}")
+
+
+def test_decode_token_chunk_scales_independent(tq):
+    """Tokens at scales 2^-120 and 2^120 in one launch, and one token whose first half
+    is 2^60 times its second: each within the parity bars of its own output."""
+    n, k, g = 136, 1024, 128
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, 4, g, seed=77)
+    xf = x.float().numpy().copy()
+    xf[0] *= np.float32(2.0 ** -120)
+    xf[1] *= np.float32(2.0 ** 120)
+    xf[2, :512] *= np.float32(2.0 ** 60)
+    xb = torch.from_numpy(xf).to(torch.bfloat16)
+    y = tq.linear_fwd(xb.cuda(), codes, s, g)
+    tq.device_status()
+    ref = O.linear_fwd(xb, w_hat)
+    for tok in range(4):
+        check_close(to_np(y[tok:tok + 1]), ref[tok:tok + 1], f"Y token {tok}")
+
+
 def test_batched_decode_mixed(tq):
     """One launch over matrices with different shapes, group sizes and output types."""
     specs = [(520, 256, 128, torch.float32), (264, 512, 32, torch.bfloat16),
