@@ -691,14 +691,21 @@ def learnable_sweep(tq, steps, warmup):
                       "frac": round(nbytes / ms / 1e6 / pk["hbm_gbs"], 4), "bytes": nbytes}
     tq.device_status()
     on, ok = OUT_PROJ
+    steps = 2000
     track = {}
-    for label, learnable in (("fixed_absmean", False), ("learnable_scale", True)):
-        rows = qat.track_zero_ratio(tq, on, ok, 1024, G, 2000, learnable, seed=5, every=400)
-        track[label] = [{kk: (round(vv, 7) if kk == "loss" else vv) for kk, vv in r.items()}
-                        for r in rows]
+    for lr in (2.5e-4, 5e-5, 1e-5):
+        per = {}
+        for label, learnable in (("fixed_absmean", False), ("learnable_scale", True)):
+            rows = qat.track_zero_ratio(tq, on, ok, 1024, G, steps, learnable, seed=5, lr=lr,
+                                        every=400)
+            per[label] = [{kk: (round(vv, 7) if kk == "loss" else vv) for kk, vv in r.items()}
+                          for r in rows]
+        track[f"lr_{lr:g}"] = per
     res["zero_ratio_tracking"] = {
         "task": f"teacher-student regression, W [{on}, {ok}] g={G}, 1024 tokens per step, "
-                "AdamW lr 2.5e-4, student from the teacher's weights",
+                f"{steps} AdamW steps (beta 0.9/0.95, decay 0.01) at each peak lr, linear "
+                f"warm-up over {steps // 50} steps then cosine decay to 0, student from the "
+                "teacher's weights",
         **track}
     return res
 

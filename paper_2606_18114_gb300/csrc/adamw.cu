@@ -199,11 +199,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           word = __any_sync(live, tiny) ? (tiny ? code_word<true>(x, s) : code_word<false>(x, s))
                                         : code_word<false>(x, s);
         }
-        const unsigned gmask =
-            kLanesPerGroup == 32 ? 0xffffffffu
-                                 : ((1u << kLanesPerGroup) - 1u) << (lane & ~(kLanesPerGroup - 1));
-        const int zc = static_cast<int>(
-            __reduce_add_sync(gmask, static_cast<unsigned>(16 - __popc(word & 0x55555555u))));
+        // zero count of the group: xor-shuffles over its lanes (a redux.sync whose
+        // mask differs between the groups of a warp is issued once per group)
+        unsigned zs = 16u - static_cast<unsigned>(__popc(word & 0x55555555u));
+        if constexpr (kLanesPerGroup == 32) {
+          zs = __reduce_add_sync(live, zs);
+        } else {
+        #pragma unroll
+          for (int off = 1; off < kLanesPerGroup; off <<= 1) zs += __shfl_xor_sync(live, zs, off);
+        }
+        const int zc = static_cast<int>(zs);
         a.codes[e >> 4] = word;
         if ((lane & (kLanesPerGroup - 1)) == 0) {
           if (kMode == kAbsmean) a.scales[e / G] = s;

@@ -17,10 +17,11 @@
 // latency (shuffle chain, reductions) needs to keep pace with HBM.
 //
 // Consumer: each lane owns 16 consecutive weights — one code word. A group
-// spans g/16 consecutive lanes; its |w| sum is reduced with log2(g/16)
-// xor-shuffles and its zero count with one redux.sync over the group's lanes (the
-// zero count of a word is 16 - popc(word & 0x5555...) because every non-zero code
-// has its low bit set).
+// spans g/16 consecutive lanes; its |w| sum and its zero count are reduced with
+// log2(g/16) xor-shuffles each (the zero count of a word is 16 - popc(word &
+// 0x5555...) because every non-zero code has its low bit set; a redux.sync over
+// the group's lanes, whose mask differs between the groups of a warp, was issued
+// once per group: 16 times per warp at g = 32).
 //
 // Code decision: see quant_code.cuh.
 #include <cuda_runtime.h>
@@ -201,11 +202,16 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
                    ? (tiny ? code_word<true>(x, tau) : code_word<false>(x, tau))
                    : code_word<false>(x, tau);
       }
-      const unsigned gmask =
-          kLanesPerGroup == 32 ? 0xffffffffu
-                               : ((1u << kLanesPerGroup) - 1u) << (lane & ~(kLanesPerGroup - 1));
-      const int zc = static_cast<int>(
-          __reduce_add_sync(gmask, static_cast<unsigned>(16 - __popc(word & 0x55555555u))));
+      // zero count of the group: xor-shuffles over its lanes (a redux.sync whose
+      // mask differs between the groups of a warp is issued once per group)
+      unsigned zs = 16u - static_cast<unsigned>(__popc(word & 0x55555555u));
+      if constexpr (kLanesPerGroup == 32) {
+        zs = __reduce_add_sync(live, zs);
+      } else {
+      #pragma unroll
+        for (int off = 1; off < kLanesPerGroup; off <<= 1) zs += __shfl_xor_sync(live, zs, off);
+      }
+      const int zc = static_cast<int>(zs);
       mt.codes[e >> 4] = word;
       if ((lane & (kLanesPerGroup - 1)) == 0) {
         if (!kGiven) mt.scales[e / G] = s;

@@ -19,24 +19,39 @@ instead and records the zero ratio as it goes:
     w from its absmean);
   - learnable scale: ds = tq_scale_grad, the scales' AdamW step (tq_adamw), then
     tq_adamw_requantize_with_scales against the new scales;
-  AdamW with the hyperparameters of §3.3 on both w and s.
+  AdamW with the hyperparameters of §3.3 on both w and s, and §3.3's schedule
+  scaled to the run's length: a linear warm-up over the first 2 % of the steps
+  (1k of 50k in the paper), then a cosine decay of the learning rate to zero.
 """
 from __future__ import annotations
 
+import math
 from typing import Dict, List
 
 import torch
 
-__all__ = ["track_zero_ratio"]
+__all__ = ["track_zero_ratio", "lr_at"]
+
+
+def lr_at(t: int, steps: int, lr: float, warmup: int) -> float:
+    """Learning rate of update t (0-based) of ``steps``: linear warm-up to ``lr`` over
+    ``warmup`` updates, then cosine decay to zero at the last update."""
+    if t < warmup:
+        return lr * (t + 1) / warmup
+    span = max(steps - warmup, 1)
+    return lr * 0.5 * (1.0 + math.cos(math.pi * (t - warmup) / span))
 
 
 def track_zero_ratio(tq, n: int, k: int, m: int, g: int, steps: int, learnable: bool,
                      seed: int = 0, lr: float = 2.5e-4, pool: int = 8,
-                     every: int = 100) -> List[Dict[str, float]]:
+                     every: int = 100, warmup: int = -1) -> List[Dict[str, float]]:
     """Run ``steps`` updates of one ternary linear layer [n, k] (group ``g``) on
-    batches of ``m`` tokens; returns ``{"step", "zero_ratio", "loss", "scale_ratio"}``
-    every ``every`` steps (and at step 0), where ``scale_ratio`` is the mean scale
-    over the mean |w| of the latent weights."""
+    batches of ``m`` tokens with peak learning rate ``lr`` (warm-up of ``warmup``
+    updates, default 2 % of ``steps``, then cosine decay); returns ``{"step",
+    "zero_ratio", "loss", "scale_ratio"}`` every ``every`` steps (and at step 0),
+    where ``scale_ratio`` is the mean scale over the mean |w| of the latent weights."""
+    if warmup < 0:
+        warmup = max(1, steps // 50)
     dev = torch.device("cuda")
     gen = torch.Generator(device=dev)
     gen.manual_seed(seed)
@@ -50,7 +65,7 @@ def track_zero_ratio(tq, n: int, k: int, m: int, g: int, steps: int, learnable: 
     y = torch.empty((m, n), device=dev)
     dw = torch.empty((n, k), device=dev)
     ds = torch.empty_like(s)
-    hp = dict(lr=lr, beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.01)
+    hp = dict(beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.01)
     out: List[Dict[str, float]] = []
     for t in range(steps + 1):
         x, y_t = xs[t % pool], ys[t % pool]
@@ -63,6 +78,7 @@ def track_zero_ratio(tq, n: int, k: int, m: int, g: int, steps: int, learnable: 
         if t == steps:
             break
         dy = (diff * (2.0 / diff.numel())).to(torch.bfloat16)
+        hp["lr"] = lr_at(t, steps, lr, warmup)
         tq.linear_bwd(dy, x, codes, s, k, g, want_dx=False, dw=dw)
         if learnable:
             tq.scale_grad(w, dw, codes, s, g, out=ds)

@@ -100,3 +100,26 @@ def test_dw_pair_schedule_sweep():
                                                [1, 2, 3, 7, 16, 64, 257]):
         if pairs <= tiles:
             _check(tiles, pairs, nkb)
+
+
+def _pieces_per_tail_tile(q):
+    return [q.owner(r * q.nkb + q.nkb - 1) - q.owner(r * q.nkb) + 1 for r in range(q.rem)]
+
+
+@pytest.mark.parametrize("m,cut", [(64, False), (1999, True), (2000, True)])
+def test_dw_stream_k_gpu_test_shapes(m, cut):
+    """The tail cases the GPU test test_dw_stream_k_tail names, for its shape
+    (n = 4160, k = 1280: 5 x 17 = 85 pair tiles) on the 76 pairs of 152 SMs: at 64
+    tokens the 9 tail tiles have fewer k-blocks than pairs and stay whole; at 1999
+    and 2000 tokens (16 k-blocks, the first ending on a ragged block) they are cut
+    into pieces, several per tile."""
+    tiles = ((1280 + 255) // 256) * ((4160 + 255) // 256)
+    nkb = (m + 127) // 128
+    q = Sched(tiles, 76, nkb)
+    assert tiles == 85
+    if not cut:
+        assert q.rem == 0
+        return
+    assert q.rem == 9 and q.units == 9 * 16
+    assert min(_pieces_per_tail_tile(q)) >= 8
+    _check(tiles, 76, nkb)

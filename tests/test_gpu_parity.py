@@ -241,14 +241,17 @@ def test_dw_accumulate_and_single_outputs(tq):
     check_close(dx2, O.linear_bwd_dx(dy, w_hat), "dX only")
 
 
-@pytest.mark.parametrize("m", [64, 640, 1000])
+@pytest.mark.parametrize("m", [64, 1999, 2000])
 @pytest.mark.parametrize("accumulate", [False, True])
 def test_dw_stream_k_tail(tq, m, accumulate):
-    """dW over more 128 x 256 tiles than SMs (10 x 17 = 170): the tiles past the last
-    whole wave are cut into runs of k-blocks, one per CTA, and summed in k order by
-    the CTA that completes each tile. m = 64 leaves fewer tail k-blocks than CTAs
-    (every tile whole), m = 640 cuts tiles into many pieces, m = 1000 ends on a
-    ragged k-block. Full comparison with the oracle."""
+    """dW over more 256 x 256 pair tiles than CTA pairs (5 x 17 = 85 tiles on the 76
+    pairs of 152 SMs): the 9 tiles past the whole wave are cut into equal runs of
+    128-token k-blocks, one run per pair, and each CTA's half of a tile is summed in
+    k order by the CTA that completes it. m = 64 leaves fewer tail k-blocks than
+    pairs (every tile whole); m = 2000 (16 k-blocks) cuts every tail tile into 8 or
+    9 pieces; m = 1999 does the same ending on a ragged k-block
+    (tests/test_dw_schedule.py checks these counts on the host). Full comparison
+    with the oracle."""
     n, k, g = 4160, 1280, 128
     w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=11, dy_std=1e-2)
     xd, dyd = x.cuda(), dy.cuda()
