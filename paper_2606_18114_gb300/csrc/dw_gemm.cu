@@ -31,10 +31,12 @@
 // barriers: a suspended waiter resumed late after an arrival from the other SM.
 //
 // Persistent: the pairs walk the tiles, k-tiles fastest, so that the pairs in
-// flight stream the same dy columns. Both operands are loaded with an L2
-// evict-last policy: x is re-read by every n-tile, and a dy block by the eight
-// pairs of its n-tile, which drift apart in token (with dy evict-first the pair
-// kernel read 1.1 GB from HBM per in_proj launch, and ran 3 % slower). Two TMEM
+// flight stream the same dy columns: a wave of 76 pair tiles covers all eight
+// k-tiles of in_proj (x, 67 MB) and 9.5 n-tiles of dy. Both operands are loaded
+// with an L2 evict-last hint (the same DRAM bytes as no hint; dy evict-first read
+// 26 % more and ran 8 % slower: the eight pairs of an n-tile drift apart in token).
+// Whole tiles alternate their token direction (see item_at), so a wave starts on
+// the x blocks the previous one read last. Two TMEM
 // accumulators (2 x 256 columns) let the epilogue of one tile overlap the main loop
 // of the next. Roles: warp 0 TMA, warp 1 MMA (leader) or relay (peer), warps 2-5
 // epilogue; the epilogue thread of lane k writes dW[n][k], so a warp store covers
@@ -106,6 +108,7 @@ struct DwItem {
   uint32_t tile;
   int kb0, kb1;  // k-blocks [kb0, kb1) of the tile
   int sk;        // -1: a whole-wave tile; else the piece's index within the pair's run
+  bool rev;      // the k-blocks are loaded last to first
 };
 
 __device__ __forceinline__ int items_of(const DwSched& q, uint32_t c) {
@@ -121,20 +124,34 @@ __device__ __forceinline__ DwItem item_at(const DwSched& q, uint32_t c, int i) {
   DwItem it;
   const int nw = q.whole_of(c);
   if (i < nw) {
+    // Whole tiles alternate their token direction, the last one running down to
+    // token 0 where the tail's pieces start: each wave begins on the x blocks that
+    // the wave before read last, which L2 still holds.
     it.tile = c + static_cast<uint32_t>(i) * q.grid;
     it.kb0 = 0;
     it.kb1 = q.nkb;
     it.sk = -1;
+    it.rev = ((nw - 1 - i) & 1) == 0;
     return it;
   }
-  const int j = i - nw;
+  // A run that crosses into the next tile takes that tile's first k-blocks before
+  // the end of the tile it starts in. Every pair then works at token offset
+  // tau + d at time tau, d in [0, nkb - run length] (0 for those first pieces, the
+  // run's start for a run inside one tile, nkb - run length for the ends), so the
+  // pairs sharing an x or dy block reach it within that window rather than up to a
+  // whole tile apart (in_proj, 44 tail tiles: 867 -> 598 MB of DRAM reads per
+  // launch). The piece keeps its index (0: the piece that opens the run) whatever
+  // the order.
   const int64_t s0 = q.run_start(c), s1 = q.run_start(c + 1);
+  const int two = (s1 - 1) / q.nkb != s0 / q.nkb;
+  const int j = two ? 1 - (i - nw) : i - nw;
   const int64_t r = s0 / q.nkb + j;  // tail tile
   const int64_t b0 = r * q.nkb;
   it.tile = q.dp + static_cast<uint32_t>(r);
   it.kb0 = static_cast<int>((s0 > b0 ? s0 : b0) - b0);
   it.kb1 = static_cast<int>((s1 < b0 + q.nkb ? s1 : b0 + q.nkb) - b0);
   it.sk = j;
+  it.rev = false;
   return it;
 }
 
@@ -211,7 +228,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           if (!(ok = mbar_wait_spin(empty_bar(s), ph ^ 1, status))) break;
           const uint32_t a = smem_base + s * kStageBytes;
           const uint32_t b = a + kABytes;
-          const int32_t mrow = kb * kKBlock;
+          const int32_t mrow = (wi.rev ? wi.kb0 + wi.kb1 - 1 - kb : kb) * kKBlock;
           mbar_arrive_expect_tx(full_bar(s), kStageBytes);
 #pragma unroll
           for (int c = 0; c < 4; ++c)  // box c: features 64 (c & 1), tokens 64 (c >> 1)

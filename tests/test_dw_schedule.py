@@ -2,8 +2,10 @@
 stream-K tail), checked for every schedule shape it can meet: each (tile, k-block) is
 computed exactly once, a split tile's pieces are contiguous and in k order, the
 fixup reads each piece from the workspace slot its writer used, no run needs more
-than its two slots, and every counter and slot index stays inside the device arrays.
-The model restates the scheduler's integer arithmetic; no GPU is involved."""
+than its two slots, every counter and slot index stays inside the device arrays, and
+the tail pieces run in the order that keeps every pair's token offset within
+nkb - (run length) of the time spent on the tail. The model restates the scheduler's
+integer arithmetic; no GPU is involved."""
 import itertools
 
 import pytest
@@ -30,11 +32,16 @@ class Sched:
         return (self.dp - 1 - c) // self.grid + 1 if c < self.dp else 0
 
     def items(self, c):
-        out = [(c + i * self.grid, 0, self.nkb, -1) for i in range(self.whole_of(c))]
+        nw = self.whole_of(c)
+        out = [(c + i * self.grid, 0, self.nkb, -1) for i in range(nw)]
+        # token direction of the whole tiles: the last one runs down to token 0
+        self.rev = [(nw - 1 - i) % 2 == 0 for i in range(nw)]
         if self.rem:
             s0, s1 = self.run_start(c), self.run_start(c + 1)
             if s1 > s0:
-                for j in range((s1 - 1) // self.nkb - s0 // self.nkb + 1):
+                npieces = (s1 - 1) // self.nkb - s0 // self.nkb + 1
+                # a run crossing into the next tile does that tile's piece first
+                for j in ([1, 0] if npieces == 2 else range(npieces)):
                     r = s0 // self.nkb + j
                     b0 = r * self.nkb
                     out.append((self.dp + r, max(s0, b0) - b0, min(s1, b0 + self.nkb) - b0, j))
@@ -58,6 +65,18 @@ def _check(tiles, pairs, nkb):
                 assert sk >= 0
                 slot_of[(c, t)] = 0 if sk == 0 else 1
     assert len(done) == tiles * nkb, "some (tile, k-block) never computed"
+    for c in range(pairs):  # directions alternate, the last whole tile ending at token 0
+        q.items(c)
+        assert all(q.rev[i] != q.rev[i + 1] for i in range(len(q.rev) - 1))
+        assert not q.rev or q.rev[-1]
+    for c in range(pairs):  # token offset minus time, over the pair's tail pieces
+        if not q.rem:
+            break
+        run = q.run_start(c + 1) - q.run_start(c)
+        tau = 0
+        for t, kb0, kb1, sk in q.items(c)[q.whole_of(c):]:
+            assert 0 <= kb0 - tau <= nkb - run, (tiles, pairs, nkb, c, q.items(c))
+            tau += kb1 - kb0
     for r in range(q.rem):
         t = q.dp + r
         b0 = r * nkb

@@ -179,6 +179,8 @@ def _setup(tq, n, k, m, g, seed=0, dy_std=1.0, dist="gauss"):
     (520, 1024, 3, 128),
     (520, 1024, 16, 128),
     (40, 64, 5, 32),         # one k-block
+    (200, 64, 300, 64),      # 256-token tiles, one forward k-block, two dX k-blocks
+    (104, 256, 400, 128),    # 256-token tiles, one dX k-block, a second half of 144 tokens
 ])
 def test_linear_parity(tq, n, k, m, g):
     w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=n + k + m)
