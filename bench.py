@@ -2,8 +2,9 @@
 
 One step = one pass of the whole path over one synthetic batch of the Mamba-2
 1.3B in_proj prefill (W fp32 [8512, 2048], g = 128, X bf16 [16384, 2048],
-dY bf16 [16384, 8512]): tq_quantize (absmean scale + ternary codes + packing),
-tq_linear_fwd (Y = X W^T), and the STE backward dX = dY W^ and dW = dY^T X.
+dY bf16 [16384, 8512]): tq_quantize_with_transpose (absmean scale + ternary codes
++ packing, and the transposed codes that dX streams, in one launch), tq_linear_fwd
+(Y = X W^T), and the STE backward dX = dY W^ and dW = dY^T X.
 ``value`` is the algorithmic TFLOP/s of the three GEMMs (3 x 2 M N K per step)
 over the device time of the whole step, inputs already in HBM; ``e2e`` is the
 same metric through the C ABI with pinned host buffers, host<->device copies of
@@ -40,9 +41,9 @@ M_PREFILL = 16384  # batch 8 x seq 2048
 G = 128
 N_LAYERS = 48
 METRIC = "W1.58A16 linear fwd+bwd TFLOP/s"
-WORKLOAD = ("Mamba-2 1.3B in_proj prefill, one step = tq_quantize W[8512,2048] (g=128) + "
-            "tq_codes_transpose + tq_linear_fwd + tq_linear_bwd (dX, dW) at M=16384 "
-            "(batch 8 x seq 2048)")
+WORKLOAD = ("Mamba-2 1.3B in_proj prefill, one step = tq_quantize_with_transpose W[8512,2048] "
+            "(g=128: codes, scales, zero counts and the transposed codes) + tq_linear_fwd + "
+            "tq_linear_bwd (dX, dW) at M=16384 (batch 8 x seq 2048)")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -284,30 +285,32 @@ class Prefill:
         n, k, g = self.n, self.k, self.g
         return n * k * 4 + n * k // 4 + 2 * 4 * n * k // g
 
+    def quantize_t_bytes(self):
+        """The fused quantize's algorithmic bytes: those of quantize and the transposed
+        codes written."""
+        return self.quantize_bytes() + self.codes_t.numel() * 4
+
     def step(self, ev=None):
         tq = self.tq
         rec = (lambda i: ev[i].record()) if ev is not None else (lambda i: None)
         rec(0)
-        tq.quantize(self.w, self.g, out=(self.codes, self.s, self.z))
+        tq.quantize_with_transpose(self.w, self.g, out=(self.codes, self.s, self.z, self.codes_t))
         rec(1)
-        tq.codes_transpose(self.codes, self.k, out=self.codes_t)
-        rec(2)
         tq.linear_fwd(self.x, self.codes, self.s, self.g, y=self.y)
-        rec(3)
+        rec(2)
         tq.linear_bwd(self.dy, self.x, self.codes, self.s, self.k, self.g, want_dw=False,
                       dx=self.dx, codes_t=self.codes_t)
-        rec(4)
+        rec(3)
         tq.linear_bwd(self.dy, self.x, self.codes, self.s, self.k, self.g, want_dx=False,
                       dw=self.dw)
-        rec(5)
+        rec(4)
 
 
 KERNELS = [  # name, source files, event span
-    ("quantize", ["quantize.cu", "ptx.cuh", "kernels.cuh"], (0, 1)),
-    ("transpose", ["quantize.cu", "kernels.cuh"], (1, 2)),
-    ("fwd", ["ts_gemm.cu", "ptx.cuh", "kernels.cuh"], (2, 3)),
-    ("dx", ["ts_gemm.cu", "ptx.cuh", "kernels.cuh"], (3, 4)),
-    ("dw", ["dw_gemm.cu", "ptx.cuh", "kernels.cuh"], (4, 5)),
+    ("quantize", ["quantize.cu", "ptx.cuh", "kernels.cuh"], (0, 1)),  # with the transpose
+    ("fwd", ["ts_gemm.cu", "ptx.cuh", "kernels.cuh"], (1, 2)),
+    ("dx", ["ts_gemm.cu", "ptx.cuh", "kernels.cuh"], (2, 3)),
+    ("dw", ["dw_gemm.cu", "ptx.cuh", "kernels.cuh"], (3, 4)),
 ]
 
 
@@ -478,7 +481,7 @@ def out_proj_step(tq, steps, warmup, shape=OUT_PROJ, act=torch.bfloat16):
     for name in ("fwd", "dx", "dw"):
         out[name] = {"ms": round(per[name], 4), "TFLOP/s": round(gemm / per[name] / 1e9, 1)}
     out["quantize"] = {"ms": round(per["quantize"], 4),
-                       "GB/s": round(p.quantize_bytes() / per["quantize"] / 1e6, 1)}
+                       "GB/s": round(p.quantize_t_bytes() / per["quantize"] / 1e6, 1)}
     del p
     return out
 
@@ -846,6 +849,8 @@ def run_only(args):
         "scale_grad": lambda: tq.scale_grad(p.w, dwr, p.codes, sg, p.g, out=ds),
         "alpha_grad": lambda: tq.alpha_grad(dwr, p.codes, p.g, out=da),
         "quantize": lambda: tq.quantize(p.w, p.g, out=(p.codes, p.s, p.z)),
+        "quantize_t": lambda: tq.quantize_with_transpose(p.w, p.g,
+                                                         out=(p.codes, p.s, p.z, p.codes_t)),
         "transpose": lambda: tq.codes_transpose(p.codes, p.k, out=p.codes_t),
         "fwd": lambda: tq.linear_fwd(p.x, p.codes, p.s, p.g, y=p.y),
         "dx": lambda: tq.linear_bwd(p.dy, p.x, p.codes, p.s, p.k, p.g, want_dw=False, dx=p.dx,
@@ -877,7 +882,7 @@ def main():
     ap.add_argument("--impl", default="tq", choices=["tq", "reference"])
     ap.add_argument("--no-extra", action="store_true", help="skip decode/quantize sweeps")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
-    ap.add_argument("--only", choices=["quantize", "transpose", "fwd", "dx", "dw", "decode", "adamw",
+    ap.add_argument("--only", choices=["quantize", "quantize_t", "transpose", "fwd", "dx", "dw", "decode", "adamw",
                                        "given", "scale_grad", "alpha_grad"],
                     help="profiling aid: run just this kernel of the step (or the batched "
                          "M=1 decode) --warmup + --steps times and print its time")
@@ -917,9 +922,8 @@ def main():
     kinfo = {}
     for name, files, _ in KERNELS:
         t = per[name]
-        if name in ("quantize", "transpose"):
-            nbytes = p.quantize_bytes() if name == "quantize" else 2 * p.n * p.k // 4
-            ach = nbytes / (t * 1e-3) / 1e9
+        if name == "quantize":
+            ach = p.quantize_t_bytes() / (t * 1e-3) / 1e9
             kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "GB/s",
                            "frac": round(ach / pk["hbm_gbs"], 4)}
         else:
@@ -928,7 +932,7 @@ def main():
                            "frac": round(ach / tc_peak, 4),
                            "frac_of_burst": round(ach / pk["bf16_tflops"], 4),
                            "frac_of_sustained": round(ach / pk["bf16_tflops_sustained"], 4)}
-    dom = max((n for n, _, _ in KERNELS if n not in ("quantize", "transpose")), key=lambda n: per[n])
+    dom = max((n for n, _, _ in KERNELS if n != "quantize"), key=lambda n: per[n])
     dom_files = dict((n, f) for n, f, _ in KERNELS)[dom]
     roof = {"kernel": dom, "bound": "tensor", "achieved": kinfo[dom]["achieved"],
             "peak": tc_peak, "unit": "TFLOP/s", "frac": kinfo[dom]["frac"],

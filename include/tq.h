@@ -93,6 +93,22 @@ TQ_API tq_status tq_quantize(const float* w, int64_t n, int64_t k, int32_t g,
                       uint32_t* codes, float* scales, int32_t* zero_counts,
                       void* stream);
 
+/*
+ * tq_quantize_with_transpose — tq_quantize, and in the same launch the transposed
+ * codes that tq_codes_transpose would make of its codes (the operand of the STE dX
+ * product on codes_t, §3.1), bit for bit the same as the two calls in a row.
+ *   w, n, k, g, codes, scales, zero_counts   as tq_quantize.
+ *   codes_t      out: uint32 [k][4 * ceil(n / 64)], layout of tq_codes_transpose;
+ *                must not overlap codes.
+ * One cooperative launch: once every CTA has written its codes (a grid barrier
+ * with the library's wait limit), the grid transposes them. A wait that runs out
+ * is reported by tq_device_status (TQ_ERR_TIMEOUT; codes_t is then incomplete).
+ * Returns TQ_ERR_CUDA if the device cannot hold the cooperative grid.
+ */
+TQ_API tq_status tq_quantize_with_transpose(const float* w, int64_t n, int64_t k, int32_t g,
+                                            uint32_t* codes, float* scales, int32_t* zero_counts,
+                                            uint32_t* codes_t, void* stream);
+
 /* Largest entry count of the batched calls. */
 #define TQ_MAX_BATCH 256
 

@@ -73,6 +73,12 @@ constexpr int kQuantMaxMats = 256;
 cudaError_t launch_quantize_batched(QuantBatch<kQuantMaxMats>& batch, int g, int* status,
                                     int num_sms, cudaStream_t stream);
 
+// launch_quantize followed, in the same cooperative launch, by launch_transpose_codes
+// of the codes it wrote.
+cudaError_t launch_quantize_t(const float* w, int64_t n, int64_t k, int g, uint32_t* codes,
+                              float* scales, int32_t* zeros, uint32_t* codes_t, int* status,
+                              int num_sms, cudaStream_t stream);
+
 // codes [n][k/16] -> codes_t [k][4 * ceil(n / 64)] (the codes of W^T).
 cudaError_t launch_transpose_codes(const uint32_t* codes, int64_t n, int64_t k, uint32_t* codes_t,
                                    cudaStream_t stream);

@@ -130,6 +130,27 @@ __device__ __forceinline__ bool mbar_wait_spin(uint32_t bar, uint32_t parity, in
   return false;
 }
 
+// Wait until the global counter *p reaches `target` (a grid barrier of a
+// cooperative launch: every CTA is resident, so every arrival comes), reading it
+// with gpu-scope acquire; gives up like mbar_wait.
+__device__ __forceinline__ bool counter_wait(const uint32_t* p, uint32_t target, int* status) {
+  uint64_t t0 = 0, limit = 0;
+  for (uint32_t n = 0;; ++n) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    if (v >= target) return true;
+    if (n == 0) {
+      t0 = globaltimer_ns();
+      limit = wait_limit_ns(status);
+    } else if ((n & 255u) == 0 && (globaltimer_ns() - t0 > limit || n >= kWaitMaxPolls)) {
+      break;
+    }
+    __nanosleep(32);
+  }
+  atomicExch(status, kStatusTimeout);
+  return false;
+}
+
 // Warp-level wait: lane 0 waits (suspended) and the outcome is broadcast; the
 // __syncwarp orders lane 0's acquire before the other lanes' reads. One waiter
 // per warp instead of 32 keeps barrier traffic off the critical path.

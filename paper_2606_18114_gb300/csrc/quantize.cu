@@ -49,6 +49,8 @@ constexpr int kSmemBytes = kStages * kStageBytes + 2 * kStages * 8 + 128;
 // flight at once.
 constexpr int kSchedSlots = 256;
 __device__ uint32_t g_sched[kSchedSlots][2];
+// Grid barrier of the fused quantize + transpose, per launch slot: {arrived, passed}.
+__device__ uint32_t g_tbar[kSchedSlots][2];
 
 // Matrix d of a batch owns the global stages [stage0, stage0 + ceil(total / kStageW));
 // a stage never spans two matrices (a matrix's last stage may be short).
@@ -61,9 +63,77 @@ __device__ __forceinline__ int find_stage_mat(const QuantMat* mats, int count, i
   return lo;
 }
 
-template <int G, int kMax, bool kGiven>
+// codes [n][k/16] -> codes_t [k][ldt]. Each thread owns one 16 x 16 block of 2-bit
+// codes (16 rows n of one code word c) and transposes it in registers with four
+// levels of block swaps (8, 4, 2, 1 fields; the two byte-sized levels are byte
+// permutes). Field p of a word holds element i(p) = 2 (p % 8) + p / 8 (the packing
+// puts the even elements in the low half), so the rows are loaded in the order
+// i(q) and the transposed word p is stored as output row i(p): the plain
+// transpose then lands every element at its packed position. Rows past n read as
+// 0, which writes the zero padding of the last words. The codes are read through
+// L2 (ld.global.cg): in the fused quantize they were written by the same launch.
+__device__ __forceinline__ void swap_fields(uint32_t& a, uint32_t& c, int shift, uint32_t mask) {
+  const uint32_t t = ((a >> shift) ^ c) & mask;
+  c ^= t;
+  a ^= t << shift;
+}
+
+__device__ __forceinline__ void transpose_block16(const uint32_t* codes, int64_t n, int64_t words,
+                                                  uint32_t* codes_t, int64_t ldt, int64_t c,
+                                                  int64_t r16) {
+  uint32_t t[16];
+#pragma unroll
+  for (int q = 0; q < 16; ++q) {
+    const int64_t row = 16 * r16 + 2 * (q & 7) + (q >> 3);
+    t[q] = row < n ? __ldcg(codes + row * words + c) : 0u;
+  }
+#pragma unroll
+  for (int w = 0; w < 8; ++w) {
+    const uint32_t a = t[w], b = t[w + 8];
+    t[w] = __byte_perm(a, b, 0x5410);
+    t[w + 8] = __byte_perm(a, b, 0x7632);
+  }
+#pragma unroll
+  for (int w = 0; w < 16; ++w) {
+    if (w & 4) continue;
+    const uint32_t a = t[w], b = t[w + 4];
+    t[w] = __byte_perm(a, b, 0x6240);
+    t[w + 4] = __byte_perm(a, b, 0x7351);
+  }
+#pragma unroll
+  for (int w = 0; w < 16; ++w)
+    if (!(w & 2)) swap_fields(t[w], t[w + 2], 4, 0x0F0F0F0Fu);
+#pragma unroll
+  for (int w = 0; w < 16; ++w)
+    if (!(w & 1)) swap_fields(t[w], t[w + 1], 2, 0x33333333u);
+  uint32_t* out = codes_t + 16 * c * ldt + r16;
+#pragma unroll
+  for (int p = 0; p < 16; ++p) out[(2 * (p & 7) + (p >> 3)) * ldt] = t[p];
+}
+
+// A warp transposes 8 consecutive words x 4 consecutive 16-row groups (32-byte
+// reads, 16-byte writes): tile `tile` of a grid of ceil(words / 8) tiles per row
+// of 4 groups.
+__device__ __forceinline__ void transpose_warp_tile(const uint32_t* codes, int64_t n, int64_t words,
+                                                    uint32_t* codes_t, int64_t ldt, int64_t tile,
+                                                    int lane) {
+  const int64_t tc = (words + 7) / 8;
+  const int64_t c = (tile % tc) * 8 + (lane & 7);
+  const int64_t r16 = (tile / tc) * 4 + (lane >> 3);
+  if (c < words && r16 < ldt) transpose_block16(codes, n, words, codes_t, ldt, c, r16);
+}
+
+// The transposed-codes output of the fused quantize (tq_quantize_with_transpose).
+struct QuantT {
+  uint32_t* codes_t;  // [k][ldt]
+  int64_t n, words, ldt;
+  uint32_t* bar;      // grid barrier of the launch: {arrived, passed}
+};
+
+template <int G, int kMax, bool kGiven, bool kT>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
-    quantize_kernel(const __grid_constant__ QuantBatch<kMax> b, uint32_t* sched, int* status) {
+    quantize_kernel(const __grid_constant__ QuantBatch<kMax> b, uint32_t* sched, int* status,
+                    const QuantT tt) {
   static_assert(G == 32 || G == 64 || G == 128 || G == 256 || G == 512, "group size");
   static_assert(kStageW % G == 0, "a group never straddles a stage");
   constexpr int kLanesPerGroup = G / 16;
@@ -154,78 +224,118 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         }
       }
     }
-    return;
+    if constexpr (!kT) return;
+  } else {
+    // ------------------------------------------------------------ consumers
+    // (a lambda: its returns end this warp's stages, not the kernel)
+    [&] {
+      int slot = 0;
+      uint32_t parity = 0;
+      // timeout tests only: this warp withholds its first "empty" arrival
+      bool withhold = blockIdx.x == 0 && warp == 0 && test_withhold(status, kWithholdQuantizeEmpty);
+      for (;;) {
+        if (!lanes_wait(full_bar(slot), parity, status)) return;
+        const int64_t ls = stage_of[slot];
+        if (ls < 0) return;
+        const QuantMat& mt = b.mats[kMax == 1 ? 0 : mat_of[slot]];
+        const int64_t total = mt.total;
+        const int64_t base = ls * kStageW + warp * kUnit;
+        const int64_t e = base + lane * 16;
+        if (e < total) {
+          // lanes of this block that hold weights; a multiple of g/16 (g | total)
+          const int64_t rem = total - base;
+          const unsigned live = rem >= kUnit ? 0xffffffffu : (1u << (rem >> 4)) - 1u;
+          const float4* src = reinterpret_cast<const float4*>(smem + slot * kStageBytes +
+                                                              (warp * kUnit + lane * 16) * 4);
+          float4 v[4];
+    #pragma unroll
+          for (int j = 0; j < 4; ++j) v[j] = src[j];
+          const float x[16] = {v[0].x, v[0].y, v[0].z, v[0].w, v[1].x, v[1].y, v[1].z, v[1].w,
+                               v[2].x, v[2].y, v[2].z, v[2].w, v[3].x, v[3].y, v[3].z, v[3].w};
+          float s = 0.f;
+          uint32_t word;
+          if constexpr (kGiven) {
+            // the learnable-scale variant: the caller's scale decides, of either sign
+            word = code_word_any(x, __ldg(mt.given_scale + e / G), live);
+          } else {
+            float sum = 0.f;
+    #pragma unroll
+            for (int j = 0; j < 4; ++j)
+              sum += (fabsf(v[j].x) + fabsf(v[j].y)) + (fabsf(v[j].z) + fabsf(v[j].w));
+    #pragma unroll
+            for (int off = 1; off < kLanesPerGroup; off <<= 1) sum += __shfl_xor_sync(live, sum, off);
+            s = sum * kInvG;  // s = (1/g) * sum |w|
+            // the decoupled quantizer decides against tau = f_row * s (one fp32 product)
+            const float tau = mt.row_factor == nullptr ? s : __fmul_rn(s, mt.row_factor[e / mt.k]);
+            // thresholds below 2^-100 (all-zero or denormal groups) take the division
+            const bool tiny = tau < 0x1p-100f;
+            word = __any_sync(live, tiny)
+                       ? (tiny ? code_word<true>(x, tau) : code_word<false>(x, tau))
+                       : code_word<false>(x, tau);
+          }
+          // zero count of the group: xor-shuffles over its lanes (a redux.sync whose
+          // mask differs between the groups of a warp is issued once per group)
+          unsigned zs = 16u - static_cast<unsigned>(__popc(word & 0x55555555u));
+          if constexpr (kLanesPerGroup == 32) {
+            zs = __reduce_add_sync(live, zs);
+          } else {
+          #pragma unroll
+            for (int off = 1; off < kLanesPerGroup; off <<= 1) zs += __shfl_xor_sync(live, zs, off);
+          }
+          const int zc = static_cast<int>(zs);
+          mt.codes[e >> 4] = word;
+          if ((lane & (kLanesPerGroup - 1)) == 0) {
+            if (!kGiven) mt.scales[e / G] = s;
+            mt.zeros[e / G] = zc;
+          }
+        }
+        __syncwarp();
+        if (lane == 0 && !withhold) mbar_arrive(empty_bar(slot));
+        withhold = false;
+        if (++slot == kStages) {
+          slot = 0;
+          parity ^= 1u;
+        }
+      }
+    }();
+    if constexpr (!kT) return;
   }
 
-  // -------------------------------------------------------------- consumers
-  int slot = 0;
-  uint32_t parity = 0;
-  // timeout tests only: this warp withholds its first "empty" arrival
-  bool withhold = blockIdx.x == 0 && warp == 0 && test_withhold(status, kWithholdQuantizeEmpty);
-  for (;;) {
-    if (!lanes_wait(full_bar(slot), parity, status)) return;
-    const int64_t ls = stage_of[slot];
-    if (ls < 0) return;
-    const QuantMat& mt = b.mats[kMax == 1 ? 0 : mat_of[slot]];
-    const int64_t total = mt.total;
-    const int64_t base = ls * kStageW + warp * kUnit;
-    const int64_t e = base + lane * 16;
-    if (e < total) {
-      // lanes of this block that hold weights; a multiple of g/16 (g | total)
-      const int64_t rem = total - base;
-      const unsigned live = rem >= kUnit ? 0xffffffffu : (1u << (rem >> 4)) - 1u;
-      const float4* src = reinterpret_cast<const float4*>(smem + slot * kStageBytes +
-                                                          (warp * kUnit + lane * 16) * 4);
-      float4 v[4];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) v[j] = src[j];
-      const float x[16] = {v[0].x, v[0].y, v[0].z, v[0].w, v[1].x, v[1].y, v[1].z, v[1].w,
-                           v[2].x, v[2].y, v[2].z, v[2].w, v[3].x, v[3].y, v[3].z, v[3].w};
-      float s = 0.f;
-      uint32_t word;
-      if constexpr (kGiven) {
-        // the learnable-scale variant: the caller's scale decides, of either sign
-        word = code_word_any(x, __ldg(mt.given_scale + e / G), live);
-      } else {
-        float sum = 0.f;
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-          sum += (fabsf(v[j].x) + fabsf(v[j].y)) + (fabsf(v[j].z) + fabsf(v[j].w));
-#pragma unroll
-        for (int off = 1; off < kLanesPerGroup; off <<= 1) sum += __shfl_xor_sync(live, sum, off);
-        s = sum * kInvG;  // s = (1/g) * sum |w|
-        // the decoupled quantizer decides against tau = f_row * s (one fp32 product)
-        const float tau = mt.row_factor == nullptr ? s : __fmul_rn(s, mt.row_factor[e / mt.k]);
-        // thresholds below 2^-100 (all-zero or denormal groups) take the division
-        const bool tiny = tau < 0x1p-100f;
-        word = __any_sync(live, tiny)
-                   ? (tiny ? code_word<true>(x, tau) : code_word<false>(x, tau))
-                   : code_word<false>(x, tau);
-      }
-      // zero count of the group: xor-shuffles over its lanes (a redux.sync whose
-      // mask differs between the groups of a warp is issued once per group)
-      unsigned zs = 16u - static_cast<unsigned>(__popc(word & 0x55555555u));
-      if constexpr (kLanesPerGroup == 32) {
-        zs = __reduce_add_sync(live, zs);
-      } else {
-      #pragma unroll
-        for (int off = 1; off < kLanesPerGroup; off <<= 1) zs += __shfl_xor_sync(live, zs, off);
-      }
-      const int zc = static_cast<int>(zs);
-      mt.codes[e >> 4] = word;
-      if ((lane & (kLanesPerGroup - 1)) == 0) {
-        if (!kGiven) mt.scales[e / G] = s;
-        mt.zeros[e / G] = zc;
+  if constexpr (kT) {
+    // Transposed codes (fused tq_codes_transpose): once every CTA has stored its
+    // stages' codes, the grid transposes them while they are still in L2. The
+    // launch is cooperative, so all CTAs are resident and the barrier completes;
+    // if it gives up, the status says so and the transpose is skipped.
+    __shared__ int passed;
+    __syncthreads();  // this CTA's code stores precede its arrival
+    if (threadIdx.x == 0) {
+      __threadfence();
+      atomicAdd(&tt.bar[0], 1u);
+      passed = counter_wait(&tt.bar[0], gridDim.x, status) ? 1 : 0;
+      // the last CTA past the barrier resets it for the next launch on this slot
+      if (atomicAdd(&tt.bar[1], 1u) == gridDim.x - 1) {
+        atomicExch(&tt.bar[0], 0u);
+        atomicExch(&tt.bar[1], 0u);
       }
     }
-    __syncwarp();
-    if (lane == 0 && !withhold) mbar_arrive(empty_bar(slot));
-    withhold = false;
-    if (++slot == kStages) {
-      slot = 0;
-      parity ^= 1u;
+    __syncthreads();
+    if (passed != 0) {
+      const int64_t tiles = ((tt.words + 7) / 8) * ((tt.ldt + 3) / 4);
+      const int64_t warps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
+      for (int64_t tile = static_cast<int64_t>(blockIdx.x) * (kThreads / 32) + warp; tile < tiles;
+           tile += warps)
+        transpose_warp_tile(b.mats[0].codes, tt.n, tt.words, tt.codes_t, tt.ldt, tile, lane);
     }
   }
+}
+
+// codes [n][k/16] -> codes_t [k][ldt], one warp per tile of 8 words x 4 groups of 16 rows.
+__global__ void __launch_bounds__(256) transpose_codes_kernel(const uint32_t* __restrict__ codes,
+                                                              int64_t n, int64_t words,
+                                                              uint32_t* __restrict__ codes_t,
+                                                              int64_t ldt, int64_t tiles) {
+  const int64_t tile = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+  if (tile < tiles) transpose_warp_tile(codes, n, words, codes_t, ldt, tile, threadIdx.x & 31);
 }
 
 // Device address of g_sched, looked up once per device.
@@ -243,88 +353,69 @@ uint32_t* sched_base() {
   return static_cast<uint32_t*>(p);
 }
 
-template <int G, int kMax, bool kGiven>
-cudaError_t launch(const QuantBatch<kMax>& b, int* status, int num_sms, cudaStream_t stream) {
-  static std::atomic<uint32_t> seq{0};
+// Device address of g_tbar, looked up once per device.
+uint32_t* tbar_base() {
+  static std::atomic<uintptr_t> base[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+  if (dev < 64) {
+    const uintptr_t p = base[dev].load(std::memory_order_acquire);
+    if (p != 0) return reinterpret_cast<uint32_t*>(p);
+  }
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_tbar) != cudaSuccess) return nullptr;
+  if (dev < 64) base[dev].store(reinterpret_cast<uintptr_t>(p), std::memory_order_release);
+  return static_cast<uint32_t*>(p);
+}
+
+std::atomic<uint32_t> g_seq{0};  // launch slot of the scheduler and the grid barrier
+
+// t.codes_t != null: the fused quantize + transpose, a cooperative launch of at
+// most the CTAs that fit on the device at once.
+template <int G, int kMax, bool kGiven, bool kT>
+cudaError_t launch(const QuantBatch<kMax>& b, int* status, int num_sms, cudaStream_t stream,
+                   QuantT t = QuantT{}) {
   if (b.nstages <= 0) return cudaSuccess;
   if (b.nstages >= (int64_t{1} << 31)) return cudaErrorInvalidValue;
-  const int64_t cap = static_cast<int64_t>(num_sms) * kCtasPerSm;
-  const int64_t blocks = b.nstages < cap ? b.nstages : cap;
-  cudaError_t e = ensure_smem_limit<quantize_kernel<G, kMax, kGiven>>(kSmemBytes);
+  auto kern = quantize_kernel<G, kMax, kGiven, kT>;
+  cudaError_t e = ensure_smem_limit<quantize_kernel<G, kMax, kGiven, kT>>(kSmemBytes);
   if (e != cudaSuccess) return e;
+  int per_sm = kCtasPerSm;
+  if (kT) {
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, kSmemBytes);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) return cudaErrorCooperativeLaunchTooLarge;
+    if (per_sm > kCtasPerSm) per_sm = kCtasPerSm;
+  }
+  const int64_t cap = static_cast<int64_t>(num_sms) * per_sm;
+  const int64_t blocks = b.nstages < cap ? b.nstages : cap;
   uint32_t* sched = sched_base();
-  if (sched == nullptr) return cudaErrorInvalidSymbol;
-  sched += 2 * (seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
-  quantize_kernel<G, kMax, kGiven><<<static_cast<unsigned>(blocks), kThreads, kSmemBytes, stream>>>(
-      b, sched, status);
-  return cudaGetLastError();
+  uint32_t* tbar = tbar_base();
+  if (sched == nullptr || tbar == nullptr) return cudaErrorInvalidSymbol;
+  const uint32_t slot = g_seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots;
+  sched += 2 * slot;
+  if (!kT) {
+    kern<<<static_cast<unsigned>(blocks), kThreads, kSmemBytes, stream>>>(b, sched, status, t);
+    return cudaGetLastError();
+  }
+  t.bar = tbar + 2 * slot;
+  void* args[] = {const_cast<QuantBatch<kMax>*>(&b), &sched, &status, &t};
+  return cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(kern),
+                                     dim3(static_cast<unsigned>(blocks)), dim3(kThreads), args,
+                                     kSmemBytes, stream);
 }
 
-template <int kMax, bool kGiven>
+template <int kMax, bool kGiven, bool kT = false>
 cudaError_t launch_g(const QuantBatch<kMax>& b, int g, int* status, int num_sms,
-                     cudaStream_t stream) {
+                     cudaStream_t stream, QuantT t = QuantT{}) {
   switch (g) {
-    case 32: return launch<32, kMax, kGiven>(b, status, num_sms, stream);
-    case 64: return launch<64, kMax, kGiven>(b, status, num_sms, stream);
-    case 128: return launch<128, kMax, kGiven>(b, status, num_sms, stream);
-    case 256: return launch<256, kMax, kGiven>(b, status, num_sms, stream);
-    case 512: return launch<512, kMax, kGiven>(b, status, num_sms, stream);
+    case 32: return launch<32, kMax, kGiven, kT>(b, status, num_sms, stream, t);
+    case 64: return launch<64, kMax, kGiven, kT>(b, status, num_sms, stream, t);
+    case 128: return launch<128, kMax, kGiven, kT>(b, status, num_sms, stream, t);
+    case 256: return launch<256, kMax, kGiven, kT>(b, status, num_sms, stream, t);
+    case 512: return launch<512, kMax, kGiven, kT>(b, status, num_sms, stream, t);
     default: return cudaErrorInvalidValue;
   }
-}
-
-// codes [n][k/16] -> codes_t [k][ldt]. Each thread owns one 16 x 16 block of 2-bit
-// codes (16 rows n of one code word c) and transposes it in registers with four
-// levels of block swaps (8, 4, 2, 1 fields; the two byte-sized levels are byte
-// permutes). Field p of a word holds element i(p) = 2 (p % 8) + p / 8 (the packing
-// puts the even elements in the low half), so the rows are loaded in the order
-// i(q) and the transposed word p is stored as output row i(p): the plain
-// transpose then lands every element at its packed position. A warp covers 8
-// consecutive words x 4 consecutive 16-row groups (32-byte reads, 16-byte writes);
-// rows past n read as 0, which writes the zero padding of the last words.
-__device__ __forceinline__ void swap_fields(uint32_t& a, uint32_t& c, int shift, uint32_t mask) {
-  const uint32_t t = ((a >> shift) ^ c) & mask;
-  c ^= t;
-  a ^= t << shift;
-}
-
-__global__ void __launch_bounds__(256) transpose_codes_kernel(const uint32_t* __restrict__ codes,
-                                                              int64_t n, int64_t k,
-                                                              uint32_t* __restrict__ codes_t,
-                                                              int64_t ldt) {
-  const int tid = threadIdx.x;
-  const int64_t c = static_cast<int64_t>(blockIdx.x) * 32 + (tid & 7) + 8 * ((tid >> 5) & 3);
-  const int64_t r16 = static_cast<int64_t>(blockIdx.y) * 8 + ((tid >> 3) & 3) + 4 * (tid >> 7);
-  const int64_t words = k >> 4;
-  if (c >= words || r16 >= ldt) return;
-  uint32_t t[16];
-#pragma unroll
-  for (int q = 0; q < 16; ++q) {
-    const int64_t row = 16 * r16 + 2 * (q & 7) + (q >> 3);
-    t[q] = row < n ? __ldg(codes + row * words + c) : 0u;
-  }
-#pragma unroll
-  for (int w = 0; w < 8; ++w) {
-    const uint32_t a = t[w], b = t[w + 8];
-    t[w] = __byte_perm(a, b, 0x5410);
-    t[w + 8] = __byte_perm(a, b, 0x7632);
-  }
-#pragma unroll
-  for (int w = 0; w < 16; ++w) {
-    if (w & 4) continue;
-    const uint32_t a = t[w], b = t[w + 4];
-    t[w] = __byte_perm(a, b, 0x6240);
-    t[w + 4] = __byte_perm(a, b, 0x7351);
-  }
-#pragma unroll
-  for (int w = 0; w < 16; ++w)
-    if (!(w & 2)) swap_fields(t[w], t[w + 2], 4, 0x0F0F0F0Fu);
-#pragma unroll
-  for (int w = 0; w < 16; ++w)
-    if (!(w & 1)) swap_fields(t[w], t[w + 1], 2, 0x33333333u);
-  uint32_t* out = codes_t + 16 * c * ldt + r16;
-#pragma unroll
-  for (int p = 0; p < 16; ++p) out[(2 * (p & 7) + (p >> 3)) * ldt] = t[p];
 }
 
 }  // namespace
@@ -478,9 +569,10 @@ cudaError_t launch_scale_grad(const float* w, const float* dw, const uint32_t* c
 
 cudaError_t launch_transpose_codes(const uint32_t* codes, int64_t n, int64_t k, uint32_t* codes_t,
                                    cudaStream_t stream) {
-  const int64_t ldt = 4 * ((n + 63) / 64);
-  dim3 grid(static_cast<unsigned>((k / 16 + 31) / 32), static_cast<unsigned>((ldt + 7) / 8));
-  transpose_codes_kernel<<<grid, 256, 0, stream>>>(codes, n, k, codes_t, ldt);
+  const int64_t ldt = 4 * ((n + 63) / 64), words = k / 16;
+  const int64_t tiles = ((words + 7) / 8) * ((ldt + 3) / 4);
+  transpose_codes_kernel<<<static_cast<unsigned>((tiles + 7) / 8), 256, 0, stream>>>(
+      codes, n, words, codes_t, ldt, tiles);
   return cudaGetLastError();
 }
 
@@ -494,6 +586,17 @@ cudaError_t launch_quantize(const float* w, int64_t n, int64_t k, int g, uint32_
   b.nstages = (n * k + kStageW - 1) / kStageW;
   return given_scale != nullptr ? launch_g<1, true>(b, g, status, num_sms, stream)
                                  : launch_g<1, false>(b, g, status, num_sms, stream);
+}
+
+cudaError_t launch_quantize_t(const float* w, int64_t n, int64_t k, int g, uint32_t* codes,
+                              float* scales, int32_t* zeros, uint32_t* codes_t, int* status,
+                              int num_sms, cudaStream_t stream) {
+  QuantBatch<1> b{};
+  b.mats[0] = QuantMat{w, codes, scales, zeros, n * k, 0, nullptr, k, nullptr};
+  b.count = 1;
+  b.nstages = (n * k + kStageW - 1) / kStageW;
+  const QuantT t{codes_t, n, k / 16, 4 * ((n + 63) / 64), nullptr};
+  return launch_g<1, false, true>(b, g, status, num_sms, stream, t);
 }
 
 cudaError_t launch_quantize_batched(QuantBatch<kQuantMaxMats>& b, int g, int* status,

@@ -358,6 +358,22 @@ TQ_API tq_status tq_quantize(const float* w, int64_t n, int64_t k, int32_t g, ui
   return e == cudaSuccess ? TQ_OK : cuda_fail(e, "quantize launch");
 }
 
+TQ_API tq_status tq_quantize_with_transpose(const float* w, int64_t n, int64_t k, int32_t g,
+                                            uint32_t* codes, float* scales, int32_t* zero_counts,
+                                            uint32_t* codes_t, void* stream) {
+  g_err[0] = 0;
+  TQ_TRY(check_quantize_args(w, n, k, g, codes, scales, zero_counts));
+  if (n == 0 || k == 0) return TQ_OK;
+  if (n > kMaxDim || k > kMaxDim) return fail(TQ_ERR_UNSUPPORTED, "dimension too large");
+  TQ_TRY(check_ptr(codes_t, "codes_t"));
+  const DeviceInfo* dev = nullptr;
+  TQ_TRY(device_info(&dev));
+  cudaError_t e = tq::launch_quantize_t(w, n, k, g, codes, scales, zero_counts, codes_t,
+                                        dev->status, dev->num_sms,
+                                        static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? TQ_OK : cuda_fail(e, "quantize + transpose launch");
+}
+
 TQ_API tq_status tq_quantize_decoupled(const float* w, int64_t n, int64_t k, int32_t g,
                                        const float* row_factor, uint32_t* codes, float* scales,
                                        int32_t* zero_counts, void* stream) {

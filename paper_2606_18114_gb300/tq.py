@@ -16,6 +16,7 @@ __all__ = [
     "TqError",
     "load",
     "quantize",
+    "quantize_with_transpose",
     "quantize_batched",
     "quant_batch",
     "linear_fwd",
@@ -46,7 +47,7 @@ IN_F16 = 0x100  # flag: fp16 activations (x, dy) instead of bf16
 STATUS = {0: "TQ_OK", 1: "TQ_ERR_INVALID_ARG", 2: "TQ_ERR_UNSUPPORTED", 3: "TQ_ERR_CUDA",
           4: "TQ_ERR_TIMEOUT"}
 # Every symbol include/tq.h declares.
-EXPORTS = ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
+EXPORTS = ("tq_quantize", "tq_quantize_with_transpose", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
            "tq_linear_bwd_noalloc", "tq_codes_transpose", "tq_linear_fwd_batched",
            "tq_adamw_requantize", "tq_quantize_decoupled", "tq_alpha_grad",
            "tq_quantize_with_scales", "tq_scale_grad", "tq_adamw_requantize_with_scales",
@@ -110,6 +111,7 @@ def load(path: Optional[str] = None):
     lib = ctypes.CDLL(p)
     i64, i32, vp = ctypes.c_int64, ctypes.c_int32, ctypes.c_void_p
     lib.tq_quantize.argtypes = [vp, i64, i64, i32, vp, vp, vp, vp]
+    lib.tq_quantize_with_transpose.argtypes = [vp, i64, i64, i32, vp, vp, vp, vp, vp]
     lib.tq_quantize_batched.argtypes = [ctypes.POINTER(QuantDesc), i32, i32, vp]
     lib.tq_linear_fwd.argtypes = [vp, i64, i64, vp, vp, i64, i32, vp, i32, vp]
     lib.tq_linear_bwd.argtypes = [vp, vp, i64, i64, i64, vp, vp, vp, i32, vp, i32, vp, i32, vp]
@@ -128,7 +130,7 @@ def load(path: Optional[str] = None):
                                                     ctypes.POINTER(AdamwHparams), vp, vp, vp, vp]
     lib.tq_adamw.argtypes = [vp, vp, vp, vp, i64, ctypes.POINTER(AdamwHparams), vp]
     lib.tq_test_hooks.argtypes = [i64, ctypes.c_uint32]
-    for name in ("tq_quantize", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
+    for name in ("tq_quantize", "tq_quantize_with_transpose", "tq_quantize_batched", "tq_linear_fwd", "tq_linear_bwd",
                  "tq_linear_bwd_noalloc", "tq_codes_transpose", "tq_linear_fwd_batched",
                  "tq_device_status", "tq_test_hooks"):
         getattr(lib, name).restype = ctypes.c_int
@@ -191,6 +193,25 @@ def quantize(w: torch.Tensor, g: int, out=None, stream=None):
     _check(load().tq_quantize(_ptr(w), n, k, g, _ptr(codes), _ptr(scales), _ptr(zeros),
                               _stream(stream)))
     return codes, scales, zeros
+
+
+def quantize_with_transpose(w: torch.Tensor, g: int, out=None, stream=None):
+    """``quantize`` and ``codes_transpose`` of its codes in one launch.
+
+    Returns ``(codes, scales, zero_counts, codes_t)``, ``codes_t`` int32
+    ``[K, 4 * ceil(N / 64)]``; ``out`` may supply all four.
+    """
+    n, k = w.shape
+    if out is None:
+        codes = torch.empty((n, k // 16), dtype=torch.int32, device=w.device)
+        scales = torch.empty((n, k // g), dtype=torch.float32, device=w.device)
+        zeros = torch.empty((n, k // g), dtype=torch.int32, device=w.device)
+        codes_t = torch.empty((k, 4 * ((n + 63) // 64)), dtype=torch.int32, device=w.device)
+    else:
+        codes, scales, zeros, codes_t = out
+    _check(load().tq_quantize_with_transpose(_ptr(w), n, k, g, _ptr(codes), _ptr(scales),
+                                             _ptr(zeros), _ptr(codes_t), _stream(stream)))
+    return codes, scales, zeros, codes_t
 
 
 def adamw_requantize(w: torch.Tensor, grad: torch.Tensor, m: torch.Tensor, v: torch.Tensor,

@@ -52,6 +52,28 @@ def test_quantize_withheld_release_times_out_then_recovers(tq):
         assert all(torch.equal(a, b) for a, b in zip(got, ref))
 
 
+def test_quantize_with_transpose_withheld_release_times_out_then_recovers(tq):
+    """The fused quantize + transpose: CTA 0 gives up on its stages and reaches the
+    grid barrier late, the others give up on the barrier; every CTA still passes the
+    barrier's reset, so after the timeout 300 clean launches (every one of the 256
+    barrier slots again) give the clean result."""
+    n, k, g = 4096, 2048, 128
+    w = torch.from_numpy(synth.latent_weights(n, k, seed=84)).cuda()
+    ref = tq.quantize_with_transpose(w, g)
+    tq.device_status()
+    try:
+        tq.test_hooks(LIMIT_NS, 1)
+        tq.quantize_with_transpose(w, g)
+        _expect_timeout(tq)
+    finally:
+        tq.test_hooks(0, 0)
+    out = tuple(torch.empty_like(t) for t in ref)
+    for _ in range(300):
+        tq.quantize_with_transpose(w, g, out=out)
+    tq.device_status()
+    assert all(torch.equal(a, b) for a, b in zip(out, ref))
+
+
 def test_dw_withheld_accumulator_times_out_then_recovers(tq):
     # in_proj shape at 640 tokens: 272 pair tiles on 76 pairs, so the first pair
     # reuses its first accumulator, and the tail tiles are cut into stream-K pieces
