@@ -528,6 +528,24 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
       for (int r = 0; r < kTiles; ++r)
 #pragma unroll
         for (int h = 0; h < 2; ++h) sp[r][h] = sl + soff[r][h] + q0;
+      // g = 128, two chunks per warp: the scales of their groups q0, q0 + 1 for all
+      // four rows, loaded once. In the unit and 16-byte modes (row strides k/g and 4,
+      // area bases on 4-group boundaries; q0 = 4s + 2kh is even) one 8-byte load per
+      // row takes both: half the loads and half the bank conflicts (a load's eight
+      // rows sit 16 or 32 words apart there). The 4-byte mode's odd row stride (5)
+      // allows no 8-byte load and has no conflicts: two 4-byte loads. Past k (last
+      // segment) the second value is not used.
+      constexpr bool kPairScales = kKind == 1 && kMine == 2;
+      float2 sv[kTiles][2];
+      if constexpr (kPairScales) {
+        const bool wide = mode != kDecodeScale4;
+#pragma unroll
+        for (int r = 0; r < kTiles; ++r)
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+            sv[r][h] = wide ? *reinterpret_cast<const float2*>(sp[r][h])
+                            : make_float2(sp[r][h][0], sp[r][h][1]);
+      }
       const uint8_t* xs = cbase + kCodeBytes + scale_bytes;  // x of the m tokens
 #pragma unroll
       for (int cc = 0; cc < kMine; ++cc) {
@@ -589,8 +607,8 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
           // C slots 0, 1: row rl + 16r, slots 2, 3: row rl + 16r + 8
 #pragma unroll
           for (int r = 0; r < kTiles; ++r) {
-            const float h0 = sp[r][0][dq];
-            const float h1 = sp[r][1][dq];
+            const float h0 = kPairScales ? (cc == 0 ? sv[r][0].x : sv[r][0].y) : sp[r][0][dq];
+            const float h1 = kPairScales ? (cc == 0 ? sv[r][1].x : sv[r][1].y) : sp[r][1][dq];
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
               acc[r][i] = fmaf(i < 2 ? h0 : h1, p[r][i], acc[r][i]);

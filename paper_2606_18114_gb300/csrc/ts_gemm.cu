@@ -52,18 +52,32 @@ constexpr int kCodesBytes = 4096;            // 128 rows x 8 code words
 // A ring, that same commit tells the expansion, kAStages iterations later, that
 // the A stage is free, otherwise a second commit goes to the A stage's barrier.
 // Tensor memory (512 columns) holds kAcc accumulators of BN columns plus the A ring:
-//   forward and dX, 256 tokens: one accumulator and four A stages (a deep A ring
-//     hides the commit -> expansion -> MMA round trip; measured against 192 tokens
-//     with two accumulators, whose epilogue overlaps the next tile, and with one
-//     accumulator and four A stages: 0.365 vs 0.373 and 0.402 ms for the in_proj
-//     forward);
+//   forward, 256 tokens ("ping-pong"): the two halves of tensor memory, 256
+//     columns each, swap roles every tile. Tile i accumulates in half i % 2 while
+//     its A ring (four stages of 64 columns, stage kb % 4 for k-block kb of the
+//     tile) lives in the other half; tile i + 1's A ring is tile i's accumulator.
+//     The epilogue drains tile i in four 64-column chunks and releases each chunk
+//     ("drained") as soon as it is in registers, before storing it; the expansion
+//     fills stage c of tile i + 1 once chunk c is released. The MMAs of the next
+//     tile so restart after a quarter of the drain instead of all of it (an fp32
+//     tile leaves the SM at ~30 B per cycle, a quarter of the tile's MMA time):
+//     in_proj forward 0.385 -> 0.379 ms alone, 0.382 -> 0.373 in the step, less
+//     than the drain's share because the stores then compete with the activation
+//     stream (~66 B per cycle into each SM) instead of pausing it. A deep A ring
+//     hides the commit -> expansion -> MMA round trip: two A stages beside a ring of
+//     three 128-token accumulator halves ran the forward in 0.411 ms;
+//   dX, 256 tokens: one accumulator and four A stages in a ring over the launch (its
+//     tiles are 67 k-blocks long at in_proj, so the drain is a small share; the
+//     ping-pong layout ran it 1 % slower);
 //   16 tokens: two accumulators and four A stages.
 template <int MODE, int BN>
 struct TsLayout {
   static_assert(BN == 16 || BN == 256, "tile tokens");
+  static constexpr bool kPingPong = BN == 256 && MODE == kTsFwd;
   static constexpr int kSmem = BN == 16 ? 16 : 3;
   static constexpr int kAStages = 4;
   static constexpr int kAcc = BN == 256 ? 1 : 2;
+  static_assert(!kPingPong || (kAcc * BN == 256 && kAStages * 64 == 256), "two halves");
   static constexpr bool kReleaseViaSmem = kSmem >= kAStages;
   static constexpr int kSubBytes = BN * 64 * 2;                // one 64-wide k half
   static constexpr int kBBytes = 2 * kSubBytes;
@@ -71,7 +85,7 @@ struct TsLayout {
   static constexpr int kScaleOff = kSmem * kStageBytes;     // dx: 2 WG x 4 warps x 2 x 64 bf16
   static constexpr int kScaleBytes = 2 * 4 * 2 * 64 * 2;
   static constexpr int kBarOff = kScaleOff + kScaleBytes;
-  static constexpr int kNumBars = 2 * kSmem + 2 * kAStages + 2 * kAcc;
+  static constexpr int kNumBars = 2 * kSmem + 2 * kAStages + 2 * kAcc + 4;  // + drained
   static constexpr int kBytes = kBarOff + kNumBars * 8 + 8;
   static constexpr int kTxBytes = kBBytes + kCodesBytes;
   static constexpr int kTmemNeed = kAcc * BN + kAStages * 64;
@@ -152,6 +166,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto aempty_bar = [&](int a) { return bar_base + 8u * (2 * kSmem + kAS + a); };
   auto accfull_bar = [&](int a) { return bar_base + 8u * (2 * kSmem + 2 * kAS + a); };
   auto accempty_bar = [&](int a) { return bar_base + 8u * (2 * kSmem + 2 * kAS + kAcc + a); };
+  // ping-pong: chunk c (64 columns) of the last tile's accumulator is in registers
+  auto drained_bar = [&](int c) { return bar_base + 8u * (2 * kSmem + 2 * kAS + 2 * kAcc + c); };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::kBarOff + L::kNumBars * 8);
 
   if (threadIdx.x == 0) {
@@ -167,6 +183,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(accfull_bar(a), 1);
       mbar_init(accempty_bar(a), 4);  // one arrival per epilogue warp
     }
+    for (int c = 0; c < 4; ++c) mbar_init(drained_bar(c), 4);  // one per epilogue warp
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -214,7 +231,36 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
-    if (lane == 0) {
+    if (L::kPingPong && lane == 0) {
+      // No wait for the accumulator: the first MMA of tile i + 1 waits for its A
+      // stage, which the expansion fills only after the epilogue has taken chunk 0
+      // of tile i, i.e. after every MMA of tile i completed (both halves are free).
+      constexpr uint32_t idesc = idesc_bf16(128, BN, 0, 0, F16);
+      int it = 0;
+      bool ok = true;
+      for (int i = 0; i < my_tiles && ok; ++i) {
+        const uint32_t d = tmem_base + 256u * (i & 1);
+        const uint32_t a0 = tmem_base + 256u * ((i + 1) & 1);
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = it % kSmem, as = kb % kAS;
+          const int use = i * ((nkb - as + kAS - 1) / kAS) + kb / kAS;  // of stage as
+          // afull implies full: the expansion warps waited on this stage's TMA
+          // barrier before they arrived, so one wait orders both operands.
+          if (!(ok = mbar_wait(afull_bar(as), use & 1, status))) break;
+          tc_fence_after();
+          const uint32_t b_addr = smem_base + s * L::kStageBytes;
+#pragma unroll
+          for (int j = 0; j < kKBlock / 16; ++j) {
+            const uint64_t bdesc =
+                smem_desc_sw128(b_addr + (j >> 2) * L::kSubBytes + (j & 3) * 32, 16, 1024);
+            mma_ts(d, a0 + as * 64 + j * 8, bdesc, idesc, (kb | j) != 0);
+          }
+          mma_commit(empty_bar(s));
+          mma_commit(aempty_bar(as));
+        }
+        if (ok) mma_commit(accfull_bar(0));
+      }
+    } else if (!L::kPingPong && lane == 0) {
       constexpr uint32_t idesc = idesc_bf16(128, BN, 0, 0, F16);
       int it = 0;
       bool ok = true;
@@ -248,6 +294,47 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quad = warp & 3;
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     const int64_t m = args.m;
+    if constexpr (L::kPingPong) {
+      for (int i = 0; i < my_tiles; ++i) {
+        if (!lanes_wait(accfull_bar(0), i & 1, status)) break;
+        tc_fence_after();
+        const int64_t row = tile_r0(i) + quad * 32 + lane;
+        const int64_t m0 = tile_m0(i);
+        const uint32_t d = tmem_base + 256u * (i & 1) + lane_off;
+        const int mvalid = static_cast<int>(m - m0 < BN ? m - m0 : BN);
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t v[4][16];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) tmem_ld16(d + 64 * c + 16 * q, v[q]);
+          tmem_ld_wait16(v[0]);
+          tmem_regs_ready16(v[1]);
+          tmem_regs_ready16(v[2]);
+          tmem_regs_ready16(v[3]);
+          // the chunk is in registers: its columns become an A stage of the next tile
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(drained_bar(c));
+          if (row < rows) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const int cc = 64 * c + 16 * q;
+              if (args.out_bf16) {
+                __nv_bfloat16* p = static_cast<__nv_bfloat16*>(args.out) + (m0 + cc) * rows + row;
+#pragma unroll
+                for (int t = 0; t < 16; ++t, p += rows)
+                  if (cc + t < mvalid) *p = __float2bfloat16_rn(__uint_as_float(v[q][t]));
+              } else {
+                float* p = static_cast<float*>(args.out) + (m0 + cc) * rows + row;
+#pragma unroll
+                for (int t = 0; t < 16; ++t, p += rows)
+                  if (cc + t < mvalid) *p = __uint_as_float(v[q][t]);
+              }
+            }
+          }
+        }
+      }
+    } else {
     for (int i = 0; i < my_tiles; ++i) {
       const int acc = i % kAcc;
       const uint32_t aph = (i / kAcc) & 1;
@@ -290,6 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(accempty_bar(acc));
     }
+    }
   } else {
     // ---------------------------------------------------------------- expansion
     // Both warpgroups take every k-block: warpgroup wg fills A columns
@@ -321,23 +409,44 @@ __global__ void __launch_bounds__(kThreads, 1)
         c.r0 = tile_r0(c.i);
       }
     };
-    // The A stage of iteration it is free once the MMAs of iteration it - kAS are done.
-    auto a_free = [&](int it) -> bool {
-      if (L::kReleaseViaSmem) {
-        if (it < kAS) return true;
-        const int j = it - kAS;
-        return lanes_wait(empty_bar(j % kSmem), (j / kSmem) & 1, status);
-      }
-      return lanes_wait(aempty_bar(it % kAS), ((it / kAS) & 1) ^ 1, status);
+    // A stage of a k-block: it % kAS in a ring over the whole launch, or (ping-pong)
+    // kb % kAS in the half of tensor memory that is not the tile's accumulator.
+    auto stage_of = [&](const Cursor& c) { return L::kPingPong ? c.kb % kAS : c.it % kAS; };
+    auto stage_col = [&](const Cursor& c) -> uint32_t {
+      if constexpr (L::kPingPong)
+        return tmem_base + 256u * ((c.i + 1) & 1) + (c.kb % kAS) * 64;
+      else
+        return tmem_a + (c.it % kAS) * 64;
     };
-    auto publish = [&](int as, const uint32_t* a) {
+    // The A stage is free once the MMAs that last read it are done: those of
+    // iteration it - kAS; ping-pong: those of k-block kb - kAS of the tile, or, for
+    // the tile's first use of the stage, the epilogue has taken the previous tile's
+    // accumulator chunk kb (those columns).
+    auto a_free = [&](const Cursor& c) -> bool {
+      if constexpr (L::kPingPong) {
+        const int as = c.kb % kAS;
+        if (c.kb < kAS) return c.i == 0 || lanes_wait(drained_bar(as), (c.i - 1) & 1, status);
+        const int use = c.i * ((nkb - as + kAS - 1) / kAS) + c.kb / kAS;  // of stage as
+        return lanes_wait(aempty_bar(as), (use - 1) & 1, status);
+      } else {
+        const int it = c.it;
+        if (L::kReleaseViaSmem) {
+          if (it < kAS) return true;
+          const int j = it - kAS;
+          return lanes_wait(empty_bar(j % kSmem), (j / kSmem) & 1, status);
+        }
+        return lanes_wait(aempty_bar(it % kAS), ((it / kAS) & 1) ^ 1, status);
+      }
+    };
+    auto publish = [&](const Cursor& c, const uint32_t* a) {
+      const uint32_t col = stage_col(c) + wg * 32 + lane_off;
       tc_fence_after();
-      tmem_st_x16(tmem_a + as * 64 + wg * 32 + lane_off, a);
-      tmem_st_x16(tmem_a + as * 64 + wg * 32 + 16 + lane_off, a + 16);
+      tmem_st_x16(col, a);
+      tmem_st_x16(col + 16, a + 16);
       tmem_st_wait();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(afull_bar(as));
+      if (lane == 0) mbar_arrive(afull_bar(stage_of(c)));
     };
     Cursor cur = cursor_at(0);
     Cursor pre = cursor_at(2);
@@ -355,7 +464,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       float2 p0 = load_sc(cur), p1 = load_sc(cursor_at(1));
       for (; cur.it < total; advance(cur), advance(pre)) {
         const int it = cur.it;
-        const int s = it % kSmem, as = it % kAS;
+        const int s = it % kSmem;
         const float2 sc = p0;
         p0 = p1;
         p1 = load_sc(pre);
@@ -371,8 +480,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         expand_word<F16>(cw.y, hs_lo, a + 8);
         expand_word<F16>(cw.z, hs_hi, a + 16);
         expand_word<F16>(cw.w, hs_hi, a + 24);
-        if (!a_free(it)) break;
-        publish(as, a);
+        if (!a_free(cur)) break;
+        publish(cur, a);
       }
     } else {
       // dX: this thread is input feature k = row; a warp shares one k-group, and
@@ -397,7 +506,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // so the expansion is the forward's with a scale pair per pair of rows n.
         for (; cur.it < total; advance(cur), advance(pre)) {
           const int it = cur.it;
-          const int s = it % kSmem, as = it % kAS;
+          const int s = it % kSmem;
           const float2 sc = p0;
           p0 = p1;
           p1 = load_sc(pre);
@@ -419,8 +528,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int j = 0; j < 8; ++j)
               a[8 * q + j] = bmul2<F16>((words[q] << (14 - 2 * j)) & 0xC000C000u, pr[j]);
           }
-          if (!a_free(it)) break;
-          publish(as, a);
+          if (!a_free(cur)) break;
+          publish(cur, a);
         }
       } else {
       // this thread's 2-bit field inside a code word of its 16-wide k slice
@@ -431,7 +540,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int xw = r_local >> 4;
       for (; cur.it < total; advance(cur), advance(pre)) {
         const int it = cur.it;
-        const int s = it % kSmem, as = it % kAS;
+        const int s = it % kSmem;
         const float2 sc = p0;
         p0 = p1;
         p1 = load_sc(pre);
@@ -451,8 +560,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t t = (__byte_perm(w0, w1, sel) << shift) & 0xC000C000u;
           a[p] = bmul2<F16>(t, spair[p]);
         }
-        if (!a_free(it)) break;
-        publish(as, a);
+        if (!a_free(cur)) break;
+        publish(cur, a);
       }
       }
     }
