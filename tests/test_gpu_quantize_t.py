@@ -47,6 +47,7 @@ def _two_calls(tq, w, g):
     (1, 512, 512),       # a single row, one stage shorter than a full one
     (130, 512, 256),
     (64, 128, 128),
+    (100, 1088, 64),     # a last 1088 % 512 = 64 columns, a ragged last row group
 ])
 def test_matches_quantize_then_transpose(tq, n, k, g):
     w = torch.from_numpy(synth.latent_weights(n, k, seed=n + k + g)).cuda()
