@@ -341,6 +341,49 @@ def time_prefill(p: Prefill, steps, warmup, world, clk=None):
     return total_ms, per
 
 
+def roofline(per, total_ms, steps, pk, pk_kind, gemm_flops, quantize_bytes):
+    """Per-kernel rates and the line's ``roofline`` object from the kernels' mean
+    CUDA-event times ``per`` (ms) inside a timed region of ``total_ms`` over ``steps``.
+
+    The measured peaks are a burst (best of 10 GEMMs) and a sustained figure (4 s of
+    back-to-back GEMMs at the power cap): a timed region of under a second takes the
+    burst peak, a longer one the sustained peak. The quantize is scored against HBM;
+    the roofline reports the slowest GEMM, with the DRAM traffic of its committed ncu
+    capture when its sources are unchanged."""
+    region_s = total_ms / 1e3
+    sustained = region_s >= 1.0
+    tc_peak = pk["bf16_tflops_sustained"] if sustained else pk["bf16_tflops"]
+    peak_rule = (f"{pk_kind} bf16 dense {'sustained' if sustained else 'burst'}: the timed region "
+                 f"({steps} steps) lasted {region_s * 1e3:.1f} ms, "
+                 f"{'at least' if sustained else 'under'} 1 s")
+    kinfo = {}
+    for name, files, _ in KERNELS:
+        t = per[name]
+        if name == "quantize":
+            ach = quantize_bytes / (t * 1e-3) / 1e9
+            kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "GB/s",
+                           "frac": round(ach / pk["hbm_gbs"], 4)}
+        else:
+            ach = gemm_flops / (t * 1e-3) / 1e12
+            kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "TFLOP/s",
+                           "frac": round(ach / tc_peak, 4),
+                           "frac_of_burst": round(ach / pk["bf16_tflops"], 4),
+                           "frac_of_sustained": round(ach / pk["bf16_tflops_sustained"], 4)}
+    dom = max((n for n, _, _ in KERNELS if n != "quantize"), key=lambda n: per[n])
+    dom_files = dict((n, f) for n, f, _ in KERNELS)[dom]
+    roof = {"kernel": dom, "bound": "tensor", "achieved": kinfo[dom]["achieved"],
+            "peak": tc_peak, "unit": "TFLOP/s", "frac": kinfo[dom]["frac"],
+            "traffic": recorded_traffic(dom, dom_files),
+            "peak_kind": peak_rule, "timed_region_ms": round(total_ms, 3),
+            "frac_of_burst": kinfo[dom]["frac_of_burst"], "burst_peak": pk["bf16_tflops"],
+            "frac_of_sustained": kinfo[dom]["frac_of_sustained"],
+            "sustained_peak": pk["bf16_tflops_sustained"],
+            "algorithmic_per_launch": gemm_flops,
+            "achieved_how": "algorithmic flops per launch / mean CUDA-event time of the "
+                            "kernel's launch inside the timed steps"}
+    return kinfo, roof
+
+
 def time_e2e(p: Prefill, steps, warmup):
     """Same step through the C ABI from pinned host buffers: every step uploads its
     inputs (W, X, dY) and reads back all its outputs (Y, dX, dW) inside the timed
@@ -909,41 +952,8 @@ def main():
     value = rate / 1e12
 
     pk, pk_kind = peaks()
-    gemm_flops = 2.0 * p.m * p.n * p.k
-    # The measured peaks are a burst (best of 10 GEMMs) and a sustained figure (4 s of
-    # back-to-back GEMMs at the power cap): a timed region of under a second takes
-    # the burst peak, a longer one the sustained peak.
-    region_s = total_ms / 1e3
-    sustained = region_s >= 1.0
-    tc_peak = pk["bf16_tflops_sustained"] if sustained else pk["bf16_tflops"]
-    peak_rule = (f"{pk_kind} bf16 dense {'sustained' if sustained else 'burst'}: the timed region "
-                 f"({args.steps} steps) lasted {region_s * 1e3:.1f} ms, "
-                 f"{'at least' if sustained else 'under'} 1 s")
-    kinfo = {}
-    for name, files, _ in KERNELS:
-        t = per[name]
-        if name == "quantize":
-            ach = p.quantize_t_bytes() / (t * 1e-3) / 1e9
-            kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "GB/s",
-                           "frac": round(ach / pk["hbm_gbs"], 4)}
-        else:
-            ach = gemm_flops / (t * 1e-3) / 1e12
-            kinfo[name] = {"ms": round(t, 4), "achieved": round(ach, 1), "unit": "TFLOP/s",
-                           "frac": round(ach / tc_peak, 4),
-                           "frac_of_burst": round(ach / pk["bf16_tflops"], 4),
-                           "frac_of_sustained": round(ach / pk["bf16_tflops_sustained"], 4)}
-    dom = max((n for n, _, _ in KERNELS if n != "quantize"), key=lambda n: per[n])
-    dom_files = dict((n, f) for n, f, _ in KERNELS)[dom]
-    roof = {"kernel": dom, "bound": "tensor", "achieved": kinfo[dom]["achieved"],
-            "peak": tc_peak, "unit": "TFLOP/s", "frac": kinfo[dom]["frac"],
-            "traffic": recorded_traffic(dom, dom_files),
-            "peak_kind": peak_rule, "timed_region_ms": round(total_ms, 3),
-            "frac_of_burst": kinfo[dom]["frac_of_burst"], "burst_peak": pk["bf16_tflops"],
-            "frac_of_sustained": kinfo[dom]["frac_of_sustained"],
-            "sustained_peak": pk["bf16_tflops_sustained"],
-            "algorithmic_per_launch": gemm_flops,
-            "achieved_how": "algorithmic flops per launch / mean CUDA-event time of the "
-                            "kernel's launch inside the timed steps"}
+    kinfo, roof = roofline(per, total_ms, args.steps, pk, pk_kind, 2.0 * p.m * p.n * p.k,
+                           p.quantize_t_bytes())
 
     e2e_steps = max(5, args.steps // 10)
     barrier(world)
