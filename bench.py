@@ -262,7 +262,7 @@ def whole_job(units_per_rank: float, world: int, max_ms: float, steps: int):
 class Prefill:
     """Device-resident inputs/outputs of one projection's prefill step."""
 
-    def __init__(self, tq, n, k, m, g, seed, act=torch.bfloat16):
+    def __init__(self, tq, n, k, m, g, seed, act=torch.bfloat16, out=torch.float32):
         gen = torch.Generator(device="cuda")
         gen.manual_seed(seed)
         self.tq, self.n, self.k, self.m, self.g = tq, n, k, m, g
@@ -273,8 +273,8 @@ class Prefill:
         self.codes_t = torch.empty((k, 4 * ((n + 63) // 64)), dtype=torch.int32, device="cuda")
         self.s = torch.empty((n, k // g), dtype=torch.float32, device="cuda")
         self.z = torch.empty((n, k // g), dtype=torch.int32, device="cuda")
-        self.y = torch.empty((m, n), dtype=torch.float32, device="cuda")
-        self.dx = torch.empty((m, k), dtype=torch.float32, device="cuda")
+        self.y = torch.empty((m, n), dtype=out, device="cuda")
+        self.dx = torch.empty((m, k), dtype=out, device="cuda")
         self.dw = torch.empty((n, k), dtype=torch.float32, device="cuda")
 
     @property
@@ -513,10 +513,10 @@ def quantize_sweep(tq, steps, warmup):
     return {"ms": round(ms, 3), "GB/s": round(nbytes / ms / 1e6, 1), "bytes": nbytes}
 
 
-def out_proj_step(tq, steps, warmup, shape=OUT_PROJ, act=torch.bfloat16):
-    """The same step on another shape (default out_proj: W [2048, 4096], X [16384, 4096])
-    or activation type."""
-    p = Prefill(tq, shape[0], shape[1], M_PREFILL, G, seed=8, act=act)
+def out_proj_step(tq, steps, warmup, shape=OUT_PROJ, act=torch.bfloat16, out=torch.float32):
+    """The same step on another shape (default out_proj: W [2048, 4096], X [16384, 4096]),
+    activation type or output type of Y and dX."""
+    p = Prefill(tq, shape[0], shape[1], M_PREFILL, G, seed=8, act=act, out=out)
     total_ms, per = time_prefill(p, steps, warmup, 1)
     ms = total_ms / steps
     gemm = 2.0 * p.m * p.n * p.k
@@ -989,6 +989,7 @@ def main():
             "quantize_48_layers_g128": quantize_sweep(tq, 5, 2),
             "out_proj_step": out_proj_step(tq, 200, 10),
             "in_proj_step_fp16_activations": out_proj_step(tq, 200, 10, IN_PROJ, torch.float16),
+            "in_proj_step_bf16_outputs": out_proj_step(tq, 200, 10, IN_PROJ, out=torch.bfloat16),
             "sweep_48_layers": g_sweep(tq),
             "adamw_requantize_g128": adamw_sweep(tq, 5, 2),
             "decoupled_in_proj": decoupled_sweep(tq, 20, 3),
