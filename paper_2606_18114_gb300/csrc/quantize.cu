@@ -24,6 +24,11 @@
 // once per group: 16 times per warp at g = 32).
 //
 // Code decision: see quant_code.cuh.
+//
+// Fused variant (tq_quantize_with_transpose): the same stages, then, in the same
+// cooperative launch, a grid barrier (a counter per launch slot, bounded wait, reset
+// by the last CTA past it) and the whole grid transposes the codes into codes_t,
+// reading them back through L2 (16 x 16 blocks, transpose_block16).
 #include <cuda_runtime.h>
 #include <stdint.h>
 
