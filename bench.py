@@ -307,7 +307,7 @@ class Prefill:
 
 
 KERNELS = [  # name, source files, event span
-    ("quantize", ["quantize.cu", "ptx.cuh", "kernels.cuh"], (0, 1)),  # with the transpose
+    ("quantize", ["quantize.cu", "ptx.cuh", "kernels.cuh", "quant_code.cuh"], (0, 1)),  # with the transpose
     ("fwd", ["ts_gemm.cu", "ptx.cuh", "kernels.cuh"], (1, 2)),
     ("dx", ["ts_gemm.cu", "ptx.cuh", "kernels.cuh"], (2, 3)),
     ("dw", ["dw_gemm.cu", "ptx.cuh", "kernels.cuh"], (3, 4)),

@@ -13,12 +13,15 @@
 // 2-D TMA load of 128-byte rows with the 128-byte swizzle (which halves the
 // consumers' bank conflicts; rows past n and columns past k read as zero;
 // narrower rows cost the TMA unit as much per row and halved the stream rate),
-// and the scales of the segment's groups a second 2-D TMA load of a box of 256
-// rows x max(4, 512/g)
-// groups that contains them (re-read from L2 by the segments sharing it; when the
-// scale rows are not a multiple of 16 bytes the producer's 32 lanes copy them
-// with 4-byte cp.async instead), both completing on the segment's "full"
-// mbarrier. TMA keeps a ring of stages
+// completing on the segment's "full" mbarrier. The group scales of a unit come
+// apart from the segments, into two buffers that alternate: with at most 32
+// groups per row the unit's rows are contiguous and arrive in one bulk copy;
+// with more, a 2-D TMA box of the unit's 256 rows x 32 groups (128-byte rows,
+// 128-byte swizzle, so that the eight rows a warp reads fall on distinct banks)
+// covers the next 32·g of k — eight segments at g = 128 — where per-segment
+// copies of each row's few scales had halved the stream. Only when the rows are
+// not a multiple of 16 bytes (k/g % 4 != 0) do the producer's 32 lanes copy each
+// segment's scales into its slot with 4-byte cp.async. TMA keeps a ring of stages
 // segments (~100 KB per SM) in flight without holding registers or load-unit
 // slots — per-lane cp.async streaming tops out near half of HBM bandwidth here.
 //
@@ -58,6 +61,7 @@
 #include <atomic>
 #include <type_traits>
 
+#include "decode.cuh"
 #include "kernels.cuh"
 #include "ptx.cuh"
 
@@ -90,21 +94,22 @@ constexpr int kMaxStages = 8;
 constexpr int kHeadBytes = 1024;                 // barriers and segment descriptors
 constexpr int kSmemLimit = 227 * 1024;
 // Slot layout (sizes set per launch from the batch's group sizes and m):
-// [codes 32 KB][scales: 256 rows x (box or segment) groups][x: m tokens x kSegK]
+// [codes 32 KB][scales: 256 rows x the segment's groups (4-byte mode only)]
+// [x: m tokens x kSegK]
 
 static_assert(kRowWarps == 8, "two m16 row tiles per row warp");
 static_assert(kCodeBytes == 32 * 1024, "codes box");
+static_assert(sizeof(DecodeBatch) <= 32764, "kernel parameter space");
+static_assert(kDecodeWinGroups * 4 == 128, "a window row is one 128-byte swizzle row");
 
 // Row strides (in floats) of the scale areas. The eight rows a warp reads at once
-// (rows = 0..7 mod 8) fall on distinct banks when the stride in 16-byte units is
-// odd, hence a 16-byte pad on rows of an even number of 16-byte units (one float
-// for the 4-byte mode) where the producer copies rows one by one. A unit's scales
-// arrive in one bulk copy and keep their rows gpr apart (per-row copies into
-// padded rows cost more than the bank conflicts they remove).
+// (rows = 0..7 mod 8) fall on distinct banks when the stride is odd, as in the
+// 4-byte mode, whose producer copies rows one by one. A unit's scales arrive in
+// one bulk copy and keep their rows gpr apart (per-row copies into padded rows
+// cost more than the bank conflicts they remove). A window's rows are 32 floats
+// apart with 16-byte chunk j of row r at chunk j ^ (r % 8) (the TMA 128-byte
+// swizzle): float q of row r sits at 32 r + (q ^ 4 (r % 8)).
 __host__ __device__ constexpr int unit_scale_stride(int gpr) { return gpr; }
-__host__ __device__ constexpr int box_scale_stride(int log2g) {
-  return decode_scale_box(log2g) % 8 == 0 ? decode_scale_box(log2g) + 4 : decode_scale_box(log2g);
-}
 __host__ __device__ constexpr int seg_scale_stride(int log2g) {
   return (log2g >= 9 ? 1 : kSegK >> log2g) | 1;
 }
@@ -189,12 +194,6 @@ __device__ __forceinline__ void mma16816_zc(float (&c)[4], uint32_t a0, uint32_t
         "{%4, %5, %6, %7}, {%8, %9}, {%10, %10, %10, %10};"
         : "=f"(c[0]), "=f"(c[1]), "=f"(c[2]), "=f"(c[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(0.0f));
-}
-
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
-               "r"(src_bytes)
-               : "memory");
 }
 
 // 4-byte global -> shared copy; zero-filled when src_bytes is 0.
@@ -291,7 +290,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     int slot = 0;
     uint32_t parity = 0;
     int64_t issued = 0;
-    int units_u = 0;  // units whose scales went through the unit buffers
+    int units_u = 0;  // units and windows whose scales went through the buffers
     bool ok = true;
     int claims = 0;
     for (;;) {
@@ -309,24 +308,41 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
       const int log2g = mt.log2g;
       const int64_t gpr = mt.k >> log2g;               // groups per row
       const int ng = log2g >= 9 ? 1 : kSegK >> log2g;  // scales per row per segment
-      if (mt.scale_mode == kDecodeScaleUnit) {
-        // all the unit's scales in one bulk copy (rows past n are not copied;
-        // their outputs are never stored)
+      // scales through the two unit buffers: the whole unit at once, or a window of
+      // kDecodeWinGroups groups (2^(log2g - 4) segments) at a time
+      const bool win = mt.scale_mode == kDecodeScaleWin;
+      // segment s opens a buffer when s & wmask == 0: every 2^(log2g - 4) segments
+      // (32 groups) in the window mode, at s = 0 in the unit mode
+      const int wmask = win ? (1 << (log2g - 4)) - 1 : 0x7fffffff;
+      auto scales_to_buffer = [&](int s) -> bool {
         const int ub = units_u & 1;
-        if (units_u >= 2 && !warp_wait(sempty_bar(ub), ((units_u >> 1) + 1) & 1, status)) {
+        if (units_u >= 2 && !warp_wait(sempty_bar(ub), ((units_u >> 1) + 1) & 1, status))
+          return false;
+        if (lane == 0) {
+          const uint32_t dst = smem_u32(ubuf + ub * ub_bytes);
+          if (win) {
+            // rows past n and groups past k/g read as zero
+            mbar_arrive_expect_tx(sfull_bar(ub), kRows * kDecodeWinGroups * 4);
+            tma_load_2d_hint(dst, &b.maps[mt.smap], sfull_bar(ub),
+                             (s >> (log2g - 4)) * kDecodeWinGroups, static_cast<int32_t>(row0),
+                             stream_policy);
+          } else {
+            // rows past n are not copied; their outputs are never stored
+            const int64_t rows = mt.n - row0 < kRows ? mt.n - row0 : kRows;
+            const uint32_t bytes = static_cast<uint32_t>(rows * gpr * 4);
+            mbar_arrive_expect_tx(sfull_bar(ub), bytes);
+            bulk_load(dst, mt.scales + row0 * gpr, bytes, sfull_bar(ub), stream_policy);
+          }
+        }
+        ++units_u;
+        return true;
+      };
+      const bool buffered = win || mt.scale_mode == kDecodeScaleUnit;
+      for (int s = 0; s < nseg; ++s) {
+        if (buffered && (s & wmask) == 0 && !scales_to_buffer(s)) {
           ok = false;
           break;
         }
-        if (lane == 0) {
-          const int64_t rows = mt.n - row0 < kRows ? mt.n - row0 : kRows;
-          const uint32_t bytes = static_cast<uint32_t>(rows * gpr * 4);
-          mbar_arrive_expect_tx(sfull_bar(ub), bytes);
-          bulk_load(smem_u32(ubuf + ub * ub_bytes), mt.scales + row0 * gpr, bytes, sfull_bar(ub),
-                    stream_policy);
-        }
-        ++units_u;
-      }
-      for (int s = 0; s < nseg; ++s) {
         if (issued >= stages && !warp_wait(empty_bar(slot), parity ^ 1u, status)) {
           ok = false;
           break;
@@ -353,36 +369,19 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
                     static_cast<const uint16_t*>(mt.x) + lane * mt.k +
                         static_cast<int64_t>(s) * kSegK,
                     xbytes, full_bar(slot), keep_policy);
-        if (mt.scale_mode == kDecodeScaleUnit) {
+        if (buffered) {
           mbar_arrive(full_bar(slot));
         } else {
-          if (mt.scale_mode == kDecodeScale16) {
-            // per row a box of sb groups from a multiple of sb, as 16-byte copies
-            // (k/g % 4 == 0 keeps them aligned), zero past n and past k
-            const int sb = decode_scale_box(log2g);
-            const int ss = box_scale_stride(log2g);
-            const int64_t gb = g0 - g0 % sb;
-            for (int i = 0; i < kRows / 32; ++i) {
-              const int r = lane + 32 * i;
-              const int64_t row = row0 + r;
-              for (int q = 0; q < sb / 4; ++q) {
-                const bool in = row < mt.n && gb + 4 * q < gpr;
-                const float* src = mt.scales + (in ? row * gpr + gb + 4 * q : 0);
-                cp_async16(sdst + (r * ss + 4 * q) * 4, src, in ? 16u : 0u);
-              }
-            }
-          } else {
-            // [256 rows][ng] from group g0 (rows seg_scale_stride apart), zero past n
-            // and past k
-            const int ss = seg_scale_stride(log2g);
-            for (int i = 0; i < kRows / 32; ++i) {
-              const int r = lane + 32 * i;
-              const int64_t row = row0 + r;
-              for (int q = 0; q < ng; ++q) {
-                const bool in = row < mt.n && g0 + q < gpr;
-                const float* src = mt.scales + (in ? row * gpr + g0 + q : 0);
-                cp_async4(sdst + (r * ss + q) * 4, src, in ? 4u : 0u);
-              }
+          // [256 rows][ng] from group g0 (rows seg_scale_stride apart), zero past n
+          // and past k
+          const int ss = seg_scale_stride(log2g);
+          for (int i = 0; i < kRows / 32; ++i) {
+            const int r = lane + 32 * i;
+            const int64_t row = row0 + r;
+            for (int q = 0; q < ng; ++q) {
+              const bool in = row < mt.n && g0 + q < gpr;
+              const float* src = mt.scales + (in ? row * gpr + g0 + q : 0);
+              cp_async4(sdst + (r * ss + q) * 4, src, in ? 4u : 0u);
             }
           }
           cp_async_arrive(full_bar(slot));
@@ -466,7 +465,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     x0_off[cc] = x_at(tok0, kh * kMine + cc);
   }
   int units_r = 0;  // units whose partial sums were handed over
-  int units_u = 0;  // units whose scales came through the unit buffers
+  int units_u = 0;  // units and windows whose scales came through the buffers
   int slot = 0;
   uint32_t parity = 0;
   for (;;) {
@@ -480,13 +479,20 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     const int log2g = si.log2g;
     const int mode = si.mode & 0xff;
     const bool unit_scales = mode == kDecodeScaleUnit;
+    const bool win_scales = mode == kDecodeScaleWin;
     const int nfull = k / kSegK;  // segments that lie inside k
     const int nseg = (k + kSegK - 1) / kSegK;
-    // Scale of unit row r and group q: area[r * sstride + q - sq0], the area being
-    // the unit buffer (sq0 = 0) or the segment's slot (sq0 = its first stored group).
+    // a window spans 2^(log2g - 4) segments (32 groups of g): segment s opens one
+    // when s & wmask == 0 and closes it when s & wmask == wmask (or s is the last)
+    const int wmask = (1 << (log2g - 4)) - 1;
+    // Scale of unit row r and group q: area[r * sstride + sq(q) - sq0], the area
+    // being the unit buffer (sq(q) = q, sq0 = 0), the segment's slot (sq(q) = q, sq0 =
+    // its first stored group) or the window buffer (sq(q) = (q & 31) ^ qx, sq0 = 0:
+    // the swizzle of row r is 4 (r % 8), and this lane's rows are all g mod 8).
     const int sstride = unit_scales ? unit_scale_stride(k >> log2g)
-                        : mode == kDecodeScale16 ? box_scale_stride(log2g)
-                                                 : seg_scale_stride(log2g);
+                        : win_scales ? kDecodeWinGroups
+                                     : seg_scale_stride(log2g);
+    const int qx = g << 2;
     const float* ubase = nullptr;
     if (unit_scales) {
       const int ub = units_u & 1;
@@ -511,30 +517,38 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     // codes are 2c, so the sums are twice the output, halved exactly at the store).
     // kKind 0 (g = 32, 64): the lane's words t and t + 4 each lie in one group,
     // whose bf16(s)/2 multiplies the expanded pairs.
-    auto segment = [&](int s, auto guard, auto kind) -> bool {
+    auto segment = [&](int s, auto guard, auto kind, auto win) -> bool {
       constexpr bool kGuard = decltype(guard)::value;
       constexpr int kKind = decltype(kind)::value;
+      constexpr bool kWin = decltype(win)::value;  // the matrix takes scale windows
+      auto sq = [&](int q) { return kWin ? (q & (kDecodeWinGroups - 1)) ^ qx : q; };
       if (s > 0 && !lanes_wait(full_bar(slot), parity, status)) return false;
+      if (kWin && (s & wmask) == 0) {
+        const int ub = units_u & 1;
+        if (!lanes_wait(sfull_bar(ub), (units_u >> 1) & 1, status)) return false;
+        ubase = reinterpret_cast<const float*>(ubuf + ub * ub_bytes);
+      }
       const uint8_t* cbase = smem + slot * slot_bytes;
       const int kseg = s * kSegK + 128 * kMine * kh;  // first k of this warp's chunks
       const int g0 = (s * kSegK) >> log2g;             // first group of the segment
-      const float* sl = unit_scales ? ubase
-                        : reinterpret_cast<const float*>(cbase + kCodeBytes) -
-                              (mode == kDecodeScale16 ? (g0 & -decode_scale_box(log2g)) : g0);
-      // scales of group q0 + dq(cc) for the lane's four rows
+      const float* sl = unit_scales || kWin
+                            ? ubase
+                            : reinterpret_cast<const float*>(cbase + kCodeBytes) - g0;
+      // scales of group q0 + dq(cc) for the lane's four rows: sp[r][h][sq(q0 + dq)]
       const float* sp[kTiles][2];
       const int q0 = kseg >> log2g;
 #pragma unroll
       for (int r = 0; r < kTiles; ++r)
 #pragma unroll
-        for (int h = 0; h < 2; ++h) sp[r][h] = sl + soff[r][h] + q0;
+        for (int h = 0; h < 2; ++h) sp[r][h] = sl + soff[r][h];
       // g = 128, two chunks per warp: the scales of their groups q0, q0 + 1 for all
-      // four rows, loaded once. In the unit and 16-byte modes (row strides k/g and 4,
-      // area bases on 4-group boundaries; q0 = 4s + 2kh is even) one 8-byte load per
-      // row takes both: half the loads and half the bank conflicts (a load's eight
-      // rows sit 16 or 32 words apart there). The 4-byte mode's odd row stride (5)
-      // allows no 8-byte load and has no conflicts: two 4-byte loads. Past k (last
-      // segment) the second value is not used.
+      // four rows, loaded once. In the unit and window modes (row strides k/g and 32,
+      // area bases on 4-group boundaries; q0 = 4s + 2kh is even, and the swizzle keeps
+      // q0 and q0 + 1 side by side) one 8-byte load per row takes both: half the loads
+      // (and, in the unit mode, half the bank conflicts: a load's eight rows sit 16 or
+      // 32 words apart there; the window's swizzle has none). The 4-byte mode's odd
+      // row stride (5) allows no 8-byte load and has no conflicts: two 4-byte loads.
+      // Past k (last segment) the second value is not used.
       constexpr bool kPairScales = kKind == 1 && kMine == 2;
       float2 sv[kTiles][2];
       if constexpr (kPairScales) {
@@ -543,8 +557,8 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
         for (int r = 0; r < kTiles; ++r)
 #pragma unroll
           for (int h = 0; h < 2; ++h)
-            sv[r][h] = wide ? *reinterpret_cast<const float2*>(sp[r][h])
-                            : make_float2(sp[r][h][0], sp[r][h][1]);
+            sv[r][h] = wide ? *reinterpret_cast<const float2*>(sp[r][h] + sq(q0))
+                            : make_float2(sp[r][h][q0], sp[r][h][q0 + 1]);
       }
       const uint8_t* xs = cbase + kCodeBytes + scale_bytes;  // x of the m tokens
 #pragma unroll
@@ -607,8 +621,8 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
           // C slots 0, 1: row rl + 16r, slots 2, 3: row rl + 16r + 8
 #pragma unroll
           for (int r = 0; r < kTiles; ++r) {
-            const float h0 = kPairScales ? (cc == 0 ? sv[r][0].x : sv[r][0].y) : sp[r][0][dq];
-            const float h1 = kPairScales ? (cc == 0 ? sv[r][1].x : sv[r][1].y) : sp[r][1][dq];
+            const float h0 = kPairScales ? (cc == 0 ? sv[r][0].x : sv[r][0].y) : sp[r][0][sq(q0 + dq)];
+            const float h1 = kPairScales ? (cc == 0 ? sv[r][1].x : sv[r][1].y) : sp[r][1][sq(q0 + dq)];
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
               acc[r][i] = fmaf(i < 2 ? h0 : h1, p[r][i], acc[r][i]);
@@ -620,10 +634,10 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
           const int qa = (kc + 16 * t) >> log2g, qb = (kc + 64 + 16 * t) >> log2g;
 #pragma unroll
           for (int r = 0; r < kTiles; ++r) {
-            const uint32_t hs0a = half_scale_x2<F16>(sl[soff[r][0] + qa]);
-            const uint32_t hs1a = half_scale_x2<F16>(sl[soff[r][1] + qa]);
-            const uint32_t hs0b = khi ? half_scale_x2<F16>(sl[soff[r][0] + qb]) : 0u;
-            const uint32_t hs1b = khi ? half_scale_x2<F16>(sl[soff[r][1] + qb]) : 0u;
+            const uint32_t hs0a = half_scale_x2<F16>(sl[soff[r][0] + sq(qa)]);
+            const uint32_t hs1a = half_scale_x2<F16>(sl[soff[r][1] + sq(qa)]);
+            const uint32_t hs0b = khi ? half_scale_x2<F16>(sl[soff[r][0] + sq(qb)]) : 0u;
+            const uint32_t hs1b = khi ? half_scale_x2<F16>(sl[soff[r][1] + sq(qb)]) : 0u;
 #pragma unroll
             for (int kb = 0; kb < 8; ++kb) {
               const int j = 2 * (kb & 3);
@@ -642,6 +656,10 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(empty_bar(slot));
+      if (kWin && ((s & wmask) == wmask || s + 1 == nseg)) {
+        if (lane == 0) mbar_arrive(sempty_bar(units_u & 1));  // after the __syncwarp
+        ++units_u;
+      }
       if (++slot == stages) {
         slot = 0;
         parity ^= 1u;
@@ -649,22 +667,28 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
       return true;
     };
     bool ok = true;
-    auto run = [&](auto kind) {
+    auto run = [&](auto kind, auto win) {
       if constexpr (kTwoTiles) {
         // (two n-tiles: no register room for a second chunk body)
-        for (int s = 0; s < nseg && ok; ++s) ok = segment(s, std::true_type{}, kind);
+        for (int s = 0; s < nseg && ok; ++s) ok = segment(s, std::true_type{}, kind, win);
       } else {
-        for (int s = 0; s < nfull && ok; ++s) ok = segment(s, std::false_type{}, kind);
-        if (ok && nfull < nseg) ok = segment(nfull, std::true_type{}, kind);
+        for (int s = 0; s < nfull && ok; ++s) ok = segment(s, std::false_type{}, kind, win);
+        if (ok && nfull < nseg) ok = segment(nfull, std::true_type{}, kind, win);
       }
+    };
+    auto run_kind = [&](auto kind) {
+      if (win_scales)
+        run(kind, std::true_type{});
+      else
+        run(kind, std::false_type{});
     };
     const bool exact = log2g >= 7;
     if (log2g == 7)
-      run(std::integral_constant<int, 1>{});
+      run_kind(std::integral_constant<int, 1>{});
     else if (exact)
-      run(std::integral_constant<int, 2>{});
+      run_kind(std::integral_constant<int, 2>{});
     else
-      run(std::integral_constant<int, 0>{});
+      run_kind(std::integral_constant<int, 0>{});
     if (!ok) return;
     if (unit_scales) {
       if (lane == 0) mbar_arrive(sempty_bar(units_u & 1));
@@ -752,7 +776,7 @@ uint32_t* dsched_base() {
 cudaError_t launch_decode(DecodeBatch& b, int num_sms, cudaStream_t stream) {
   static std::atomic<uint32_t> seq{0};
   // longest rows first: the units claimed last are the shortest (matrices and
-  // their tensor maps move together)
+  // their code maps move together; the scale maps above count stay where they are)
   int order[kDecodeMaxMats];
   for (int d = 0; d < b.count; ++d) order[d] = d;
   std::stable_sort(order, order + b.count,
@@ -779,8 +803,9 @@ cudaError_t launch_decode(DecodeBatch& b, int num_sms, cudaStream_t stream) {
   b.total_units = static_cast<int32_t>(units);
   if (b.total_units <= 0) return cudaSuccess;
   const int64_t blocks = units < num_sms ? units : num_sms;
-  // unit-scale buffers: the largest unit of scales among unit-mode matrices;
-  // ring slot: codes + the widest per-segment scale area + x of the m tokens
+  // scale buffers: the largest unit of scales among unit-mode matrices, a window
+  // (256 rows x 32 groups, 1024-byte aligned for the swizzle) if any matrix takes
+  // windows; ring slot: codes + the widest per-segment scale area + x of the m tokens
   int64_t ugroups = 0;
   int sgroups = 0;
   for (int d = 0; d < b.count; ++d) {
@@ -789,8 +814,10 @@ cudaError_t launch_decode(DecodeBatch& b, int num_sms, cudaStream_t stream) {
     if (b.mats[d].scale_mode == kDecodeScaleUnit) {
       const int64_t w = unit_scale_stride(static_cast<int>(gpr));  // gpr <= 32 in this mode
       ugroups = w > ugroups ? w : ugroups;
+    } else if (b.mats[d].scale_mode == kDecodeScaleWin) {
+      ugroups = kDecodeWinGroups;  // the most a unit-mode matrix takes too
     } else {
-      const int w = b.mats[d].scale_mode == kDecodeScale16 ? box_scale_stride(lg) : seg_scale_stride(lg);
+      const int w = seg_scale_stride(lg);
       sgroups = w > sgroups ? w : sgroups;
     }
   }

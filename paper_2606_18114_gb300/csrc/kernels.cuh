@@ -140,49 +140,7 @@ cudaError_t launch_ts_gemm(int mode, int bn, const CUtensorMap& tmap_b,
                            const CUtensorMap& tmap_codes, const TsArgs& args, int num_sms,
                            cudaStream_t stream);
 
-// decode.cu ------------------------------------------------------------------
-// Forward for m <= 16 tokens over one or many matrices in one launch.
-struct DecodeMat {
-  const float* scales;    // fp32 [n][k/g]
-  const void* x;          // bf16 [m][k]
-  void* y;                // [m][n], fp32 or bf16
-  int64_t n, k;           // k % 64 == 0
-  int32_t log2g;
-  int32_t y_bf16;
-  int32_t unit0;          // first unit of this matrix in the batch (set by the launcher)
-  int32_t scale_mode;     // how the kernel fetches scales (host-set, kDecodeScale*)
-};
-
-// Scale fetch modes: per segment in 4-byte pieces; per segment in 16-byte pieces
-// (k/g % 4 == 0); a whole unit in one bulk copy (k/g % 4 == 0, k/g <= 32).
-constexpr int kDecodeScale4 = 0, kDecodeScale16 = 1, kDecodeScaleUnit = 2;
-constexpr int kDecodeMaxMats = 128;  // per launch (the tensor maps travel as parameters)
-constexpr int kDecodeRows = 256;    // weight rows per work unit
-constexpr int kDecodeSegK = 512;    // k per streamed segment (128-byte code rows)
-
-// Groups per row of a decode scale box: kDecodeSegK / g, at least 4 (16 bytes).
-__host__ __device__ constexpr int decode_scale_box(int log2g) {
-  return (kDecodeSegK >> log2g) > 4 ? (kDecodeSegK >> log2g) : 4;
-}
-
-struct DecodeBatch {
-  // codes of matrix d as uint32 [n][k/16], box {kDecodeSegK / 16 words, kDecodeRows rows},
-  // 128-byte swizzle
-  CUtensorMap maps[kDecodeMaxMats];
-  DecodeMat mats[kDecodeMaxMats];
-  int* status;            // device status word (timeouts)
-  int32_t count;
-  int32_t m;              // tokens, 1..16
-  int32_t total_units;    // sum over matrices of ceil(n / kDecodeRows) (set by the launcher)
-  int32_t slot_bytes;     // shared-memory ring slot: codes, scales, x (set by the launcher)
-  int32_t scale_bytes;    // scale area of a slot
-  int32_t stages;         // ring slots
-  int32_t ubuf_bytes;     // one unit-scale buffer (two are kept)
-  int32_t in_f16;         // 1: fp16 activations in every matrix (else bf16)
-};
-
-// Reorders b.mats / b.maps (decreasing k) and sets unit0 and total_units.
-cudaError_t launch_decode(DecodeBatch& batch, int num_sms, cudaStream_t stream);
+// decode.cu: declared in decode.cuh.
 
 // dw_gemm.cu -----------------------------------------------------------------
 // dW[n][k] (+)= sum_m dy[m][n] x[m][k], both operands MN-major from TMA.

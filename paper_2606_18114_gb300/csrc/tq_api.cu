@@ -16,6 +16,7 @@
 #include <mutex>
 #include <unordered_map>
 
+#include "decode.cuh"
 #include "kernels.cuh"
 #include "tq.h"
 
@@ -223,7 +224,7 @@ struct MapKeyHash {
 };
 
 // kind 0: codes uint32 [n][k/16]; kind 1: scales fp32 [n][k/g] (k here = k/g) with
-// a box of `box` groups.
+// a box of `box` groups (128 bytes: the 128-byte swizzle) x kDecodeRows rows.
 tq_status decode_map(int kind, const void* base, int64_t n, int64_t k, uint32_t box,
                      CUtensorMap* out) {
   static std::mutex mu;
@@ -245,7 +246,7 @@ tq_status decode_map(int kind, const void* base, int64_t n, int64_t k, uint32_t 
                     tq::kDecodeSegK / 16, tq::kDecodeRows, CU_TENSOR_MAP_SWIZZLE_128B));
   else
     TQ_TRY(make_map(out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, base, k, n, box, tq::kDecodeRows,
-                    CU_TENSOR_MAP_SWIZZLE_NONE));
+                    CU_TENSOR_MAP_SWIZZLE_128B));
   std::lock_guard<std::mutex> lock(mu);
   if (cache.size() >= 4096) cache.clear();
   cache.emplace(key, *out);
@@ -259,7 +260,7 @@ tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
   const DeviceInfo* dev = nullptr;
   TQ_TRY(device_info(&dev));
   thread_local tq::DecodeBatch b;
-  int used = 0;
+  int used = 0, used_smaps = 0;
   // one activation type per call (checked by the callers)
   b.in_f16 = count > 0 && in_f16(descs[0].y_dtype);
   auto flush = [&]() -> tq_status {
@@ -269,6 +270,7 @@ tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
     b.m = static_cast<int32_t>(m);
     b.total_units = 0;
     used = 0;
+    used_smaps = 0;
     cudaError_t e = tq::launch_decode(b, dev->num_sms, stream);
     return e == cudaSuccess ? TQ_OK : cuda_fail(e, "decode launch");
   };
@@ -285,6 +287,12 @@ tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
     if (d.k > (int64_t(1) << 30)) return fail(TQ_ERR_UNSUPPORTED, "decode reduction longer than 2^30");
     const int log2g = log2_group(d.g);
     const int64_t gpr = d.k >> log2g;
+    const int mode = gpr % 4 != 0                 ? tq::kDecodeScale4
+                     : gpr <= tq::kDecodeWinGroups ? tq::kDecodeScaleUnit
+                                                   : tq::kDecodeScaleWin;
+    // code maps from the bottom of maps[], window-mode scale maps from the top
+    const int nmaps = mode == tq::kDecodeScaleWin ? 2 : 1;
+    if (used + used_smaps + nmaps > tq::kDecodeMaxMats) TQ_TRY(flush());
     TQ_TRY(decode_map(0, d.codes, d.n, d.k, 0, &b.maps[used]));
     tq::DecodeMat& dm = b.mats[used++];
     dm.scales = d.scales;
@@ -295,10 +303,13 @@ tq_status decode_checked(const tq_fwd_desc* descs, int32_t count, int64_t m,
     dm.log2g = log2g;
     dm.y_bf16 = out_type(d.y_dtype) == TQ_OUT_BF16;
     dm.unit0 = 0;
-    dm.scale_mode = gpr % 4 != 0 ? tq::kDecodeScale4
-                    : gpr <= 32  ? tq::kDecodeScaleUnit
-                                 : tq::kDecodeScale16;
-    if (used == tq::kDecodeMaxMats) TQ_TRY(flush());
+    dm.scale_mode = static_cast<int16_t>(mode);
+    dm.smap = 0;
+    if (mode == tq::kDecodeScaleWin) {
+      // rows of k/g floats (a multiple of 16 bytes), scales 16-byte aligned (checked)
+      dm.smap = tq::kDecodeMaxMats - 1 - used_smaps++;
+      TQ_TRY(decode_map(1, d.scales, d.n, gpr, tq::kDecodeWinGroups, &b.maps[dm.smap]));
+    }
   }
   return flush();
 }

@@ -458,6 +458,48 @@ def test_decode_long_reduction(tq, m):
     check_close(to_np(y), O.linear_fwd(x, w_hat), f"Y m={m} k={k}")
 
 
+# k/g > 32 with k/g % 4 == 0: the scales arrive in windows of 32 groups of all the
+# unit's rows (256 x 128 bytes, swizzled); each k ends inside a window (a partial last
+# window whose groups past k/g read as zero).
+_WINDOW_K = {32: 1664, 64: 2816, 128: 4608, 256: 9216, 512: 18432}  # k/g = 52, 44, 36, 36, 36
+
+
+@pytest.mark.parametrize("g", [32, 64, 128, 256, 512])
+@pytest.mark.parametrize("m", [1, 8, 9, 16])
+def test_decode_scale_windows(tq, g, m):
+    """Decode with the group scales in windows: every g, one to sixteen tokens, a
+    ragged last unit (300 rows = 256 + 44)."""
+    n, k = 300, _WINDOW_K[g]
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=900 + g + m)
+    y = tq.linear_fwd(x.cuda(), codes, s, g)
+    tq.device_status()
+    check_close(to_np(y), O.linear_fwd(x, w_hat), f"Y windows g={g} m={m}")
+
+
+def test_batched_decode_scale_modes_past_the_map_limit(tq):
+    """One call over 70 window-mode matrices (two tensor maps each: more than one
+    launch holds, so the call splits) mixed with unit-mode (k/g <= 32) and 4-byte-mode
+    (k/g % 4 != 0) matrices, fp32 and bf16 outputs."""
+    g, m = 128, 3
+    specs = [(16 + 8 * (i % 5), 4608 if i % 2 else 8192) for i in range(70)]
+    specs[10:10] = [(264, 1024), (40, 1152)]    # unit mode (k/g 8), 4-byte mode (k/g 9)
+    specs.append((520, 640))                    # 4-byte mode (k/g 5)
+    items = []
+    for i, (n, k) in enumerate(specs):
+        w = synth.latent_weights(n, k, seed=3000 + i)
+        x = synth.activations_bf16(m, k, seed=3000 + i)
+        codes, s, z = _quant(tq, w, g)
+        dt = torch.bfloat16 if i % 3 == 0 else torch.float32
+        items.append(dict(x=x.cuda(), codes=codes, scales=s, g=g,
+                          y=torch.empty((m, n), device="cuda", dtype=dt),
+                          ref=O.linear_fwd(x, validated_w_hat(w, g, codes, s, z))))
+    tq.linear_fwd_batched(items, m)
+    tq.device_status()
+    for i, it in enumerate(items):
+        check_close(it["y"].float(), it["ref"], f"batched Y[{i}] {specs[i]}",
+                    max_rel_rms=3e-2 if it["y"].dtype == torch.bfloat16 else 2e-2)
+
+
 def test_prefill_few_rows_many_tokens(tq):
     """64 weight rows (half a tile) against 40000 tokens (157 token tiles with a
     ragged last one), all three products."""
