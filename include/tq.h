@@ -270,7 +270,11 @@ TQ_API tq_status tq_adamw(float* p, const float* grad, float* m, float* v, int64
  *   the codes on chip and accumulate in fp32 (the decode kernel folds the fp32
  *   scale into each group's sum for g >= 128, the others multiply the expanded
  *   codes by bf16(s)). The decode kernel takes k <= 2^30 and n < 2^31
- *   (TQ_ERR_UNSUPPORTED beyond).
+ *   (TQ_ERR_UNSUPPORTED beyond). When a decode launch has fewer blocks of 256
+ *   rows than the device has SMs, it cuts k into 2, 4 or 8 pieces, each block's
+ *   pieces run by one thread-block cluster whose first CTA adds the others'
+ *   partial sums to its own in piece order: the same result on every run (its
+ *   rounding differs from that of an uncut launch by the order of the sums).
  */
 TQ_API tq_status tq_linear_fwd(const void* x, int64_t m, int64_t k,
                         const uint32_t* codes, const float* scales, int64_t n, int32_t g,

@@ -59,6 +59,7 @@
 
 #include <algorithm>
 #include <atomic>
+#include <mutex>
 #include <type_traits>
 
 #include "decode.cuh"
@@ -81,6 +82,22 @@ struct DecodeCfg {
   static constexpr int kThreads = (kConsumers + 1) * 32;  // + one producer warp
 };
 constexpr int kRedBytes = 2 * kRowWarps * 32 * kTiles * 4 * 4;  // partial sums, two units
+// Launches that cut k into P pieces: the first CTA of a cluster receives the
+// partial sums of the other P - 1, [piece - 1][row warp][lane][8 floats, or 16
+// with two n-tiles].
+template <bool kTwoTiles>
+__host__ __device__ constexpr int xpart_lane_floats() { return kTwoTiles ? 16 : 8; }
+// Bytes one CTA sends for one row warp: 32 (two float4, one per row tile) from
+// each of the 8 lanes of every t with tokens 2t, 2t + 1 below m, and as much for
+// tokens 8 + 2t, 9 + 2t with two n-tiles.
+template <bool kTwoTiles>
+__host__ __device__ constexpr int xpart_slice_bytes(int m) {
+  return 8 * 32 * (((m < 8 ? m : 8) + 1) / 2 +
+                   (kTwoTiles && m > 8 ? (m - 8 + 1) / 2 : 0));
+}
+__host__ __device__ constexpr int xpart_bytes(bool two_tiles, int pieces) {
+  return pieces > 1 ? (pieces - 1) * kRowWarps * 32 * (two_tiles ? 16 : 8) * 4 : 0;
+}
 // (the hand-off area exists only where two warps share a row slice)
 template <bool kTwoTiles>
 __host__ __device__ constexpr int red_bytes() { return kTwoTiles ? 0 : kRedBytes; }
@@ -121,7 +138,7 @@ struct SegInfo {
   int32_t mat;    // matrix of the batch; -1: end of the stream
   int32_t row0;   // first row of the unit
   int32_t seg;    // segment index along k
-  int32_t last;   // last segment of the unit
+  int32_t s1;     // end of the unit's segments (exclusive; its first is seg of its first stage)
   int32_t k;      // reduction length
   int32_t n;      // rows of the matrix
   int32_t log2g;
@@ -219,6 +236,63 @@ __device__ __forceinline__ uint32_t half_scale_x2(float s) {
   return u | (u << 16);
 }
 
+// Wait, with cluster-scope acquire, for a phase completed by arrivals from other
+// CTAs of the cluster (mbar_arrive_remote, a cluster-scope release), so that this
+// thread's later reads of their shared memory see what they wrote before
+// arriving. Gives up like mbar_wait.
+__device__ __forceinline__ bool mbar_test_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ bool lanes_wait_cluster(uint32_t bar, uint32_t parity, int* status) {
+  bool ok = mbar_test_wait_cluster(bar, parity);
+  if (!ok) {
+    const uint64_t t0 = globaltimer_ns();
+    const uint64_t limit = wait_limit_ns(status);
+    for (uint32_t n = 1;; ++n) {
+      if (mbar_test_wait_cluster(bar, parity)) {
+        ok = true;
+        break;
+      }
+      if ((n & 255u) == 0 && (globaltimer_ns() - t0 > limit || n >= kWaitMaxPolls)) {
+        atomicExch(status, kStatusTimeout);
+        break;
+      }
+    }
+  }
+  return __all_sync(0xffffffffu, ok);
+}
+
+// The cluster barrier in two halves: every thread arrives once the barriers are
+// set up; a warp about to touch another CTA's shared memory waits for all
+// arrivals, which also means that every CTA has started.
+__device__ __forceinline__ void cluster_arrive() {
+  // relaxed: the barrier set-up it covers was released by fence.mbarrier_init
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// 16 bytes into another CTA's shared memory, counted on that CTA's mbarrier
+// (addresses from map_to_rank): the barrier's phase completes once all the bytes
+// it expects have landed.
+__device__ __forceinline__ void st_async_f4(uint32_t cluster_addr, float4 v, uint32_t cluster_bar) {
+  asm volatile(
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+          cluster_addr),
+      "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(cluster_bar)
+      : "memory");
+}
+
 // Binary search: matrix d with unit0[d] <= u < unit0[d + 1].
 __device__ __forceinline__ int find_mat(const DecodeBatch& b, int u) {
   int lo = 0, hi = b.count - 1;
@@ -235,7 +309,9 @@ __device__ __forceinline__ int find_mat(const DecodeBatch& b, int u) {
 constexpr int kSchedSlots = 256;
 __device__ uint32_t g_dsched[kSchedSlots][2];
 
-template <bool kTwoTiles, bool F16>
+// kPieces: a launch that cuts k into pieces (clusters; b.pieces > 1); without it
+// the persistent grid, compiled with none of the pieces' code.
+template <bool kTwoTiles, bool F16, bool kPieces>
 __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     decode_kernel(const __grid_constant__ DecodeBatch b, uint32_t* sched) {
   constexpr int kConsumers = DecodeCfg<kTwoTiles>::kConsumers;
@@ -244,7 +320,9 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
   uint8_t* head = align_shared<1024>(smem_raw);
   const int ub_bytes = b.ubuf_bytes;       // one unit-scale buffer (0: none in this launch)
   float* red = reinterpret_cast<float*>(head + kHeadBytes);  // [2][kRowWarps][32][8]
-  uint8_t* ubuf = head + kHeadBytes + red_bytes<kTwoTiles>();  // two unit-scale buffers
+  const int pieces = kPieces ? b.pieces : 1;  // pieces of k per block of rows (cluster size)
+  float* xpart = reinterpret_cast<float*>(head + kHeadBytes + red_bytes<kTwoTiles>());
+  uint8_t* ubuf = reinterpret_cast<uint8_t*>(xpart) + xpart_bytes(kTwoTiles, pieces);
   uint8_t* smem = ubuf + 2 * ub_bytes;     // the ring
   const int stages = b.stages;
   const int slot_bytes = b.slot_bytes;
@@ -258,6 +336,10 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
   // partial-sum hand-off between the two warps of a row slice, per buffer
   auto rfull_bar = [&](int w, int p) { return bars + 160 + 8 * (2 * w + p); };
   auto rempty_bar = [&](int w, int p) { return bars + 288 + 8 * (2 * w + p); };
+  // pieces of k: in the first CTA of a cluster, "the other CTAs' partial sums of
+  // row warp w are written"; in the others, "the first CTA has read them"
+  auto xfull_bar = [&](int w) { return bars + 416 + 8 * w; };
+  auto xdone_bar = [&](int w) { return bars + 896 + 8 * w; };
   SegInfo* info = reinterpret_cast<SegInfo*>(head + 512);  // kMaxStages x 48 bytes
   int* status = b.status;
 
@@ -279,9 +361,20 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
         mbar_init(rfull_bar(w, p), 1);
         mbar_init(rempty_bar(w, p), 1);
       }
+    if (pieces > 1)
+      for (int w = 0; w < kRowWarps; ++w) {
+        // completed by the bytes the other CTAs store (the one arrival is this one)
+        mbar_init(xfull_bar(w), 1);
+        mbar_arrive_expect_tx(xfull_bar(w), (pieces - 1) * xpart_slice_bytes<kTwoTiles>(m));
+        mbar_init(xdone_bar(w), 1);
+      }
     fence_mbar_init();
   }
   __syncthreads();
+  // Every CTA of the cluster has started and set up its barriers once the cluster
+  // barrier completes: arrive now, wait only before the first access to another
+  // CTA's shared memory (long since complete by then).
+  if (pieces > 1) cluster_arrive();
 
   if (warp == kConsumers) {
     // ------------------------------------------------------------ producer
@@ -295,24 +388,32 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     int claims = 0;
     for (;;) {
       // the first unit of every CTA is dealt (blocks <= units), later ones claimed
+      // (with pieces of k every CTA takes its one dealt unit)
       int u = static_cast<int>(blockIdx.x);
       if (claims++ > 0) {
+        if (pieces > 1) break;
         if (lane == 0) u = static_cast<int>(gridDim.x + atomicAdd(&sched[0], 1u));
         u = __shfl_sync(0xffffffffu, u, 0);
       }
       if (u >= b.total_units) break;
       const int d = find_mat(b, u);
       const DecodeMat& mt = b.mats[d];
-      const int64_t row0 = static_cast<int64_t>(u - mt.unit0) * kRows;
       const int nseg = static_cast<int>((mt.k + kSegK - 1) / kSegK);
+      // unit = (block of rows, piece of k): piece p of P takes segments
+      // [p nseg / P, (p + 1) nseg / P), none empty (the launcher keeps P <= nseg)
+      const int local = u - mt.unit0;
+      const int piece = local % pieces;
+      const int64_t row0 = static_cast<int64_t>(local / pieces) * kRows;
+      const int s0 = piece * nseg / pieces, s1 = (piece + 1) * nseg / pieces;
       const int log2g = mt.log2g;
       const int64_t gpr = mt.k >> log2g;               // groups per row
       const int ng = log2g >= 9 ? 1 : kSegK >> log2g;  // scales per row per segment
       // scales through the two unit buffers: the whole unit at once, or a window of
       // kDecodeWinGroups groups (2^(log2g - 4) segments) at a time
       const bool win = mt.scale_mode == kDecodeScaleWin;
-      // segment s opens a buffer when s & wmask == 0: every 2^(log2g - 4) segments
-      // (32 groups) in the window mode, at s = 0 in the unit mode
+      // segment s opens a buffer at the unit's first segment and, in the window
+      // mode, when s & wmask == 0 (windows of 32 groups from group 0, every
+      // 2^(log2g - 4) segments)
       const int wmask = win ? (1 << (log2g - 4)) - 1 : 0x7fffffff;
       auto scales_to_buffer = [&](int s) -> bool {
         const int ub = units_u & 1;
@@ -338,8 +439,8 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
         return true;
       };
       const bool buffered = win || mt.scale_mode == kDecodeScaleUnit;
-      for (int s = 0; s < nseg; ++s) {
-        if (buffered && (s & wmask) == 0 && !scales_to_buffer(s)) {
+      for (int s = s0; s < s1; ++s) {
+        if (buffered && (s == s0 || (s & wmask) == 0) && !scales_to_buffer(s)) {
           ok = false;
           break;
         }
@@ -356,7 +457,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
                                ? mt.k - static_cast<int64_t>(s) * kSegK : kSegK;
         const uint32_t xbytes = static_cast<uint32_t>(kx) * 2u;
         if (lane == 0) {
-          info[slot] = SegInfo{d, static_cast<int32_t>(row0), s, s + 1 == nseg ? 1 : 0,
+          info[slot] = SegInfo{d, static_cast<int32_t>(row0), s, s1,
                                static_cast<int32_t>(mt.k), static_cast<int32_t>(mt.n),
                                log2g, mt.scale_mode | (mt.y_bf16 << 8), mt.y, 0};
           mbar_arrive_expect_tx(full_bar(slot), kCodeBytes + static_cast<uint32_t>(m) * xbytes);
@@ -481,7 +582,9 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     const bool unit_scales = mode == kDecodeScaleUnit;
     const bool win_scales = mode == kDecodeScaleWin;
     const int nfull = k / kSegK;  // segments that lie inside k
-    const int nseg = (k + kSegK - 1) / kSegK;
+    // this unit's piece of the segments (all of them without pieces)
+    const int s0 = kPieces ? si.seg : 0;
+    const int s1 = kPieces ? si.s1 : (k + kSegK - 1) / kSegK;
     // a window spans 2^(log2g - 4) segments (32 groups of g): segment s opens one
     // when s & wmask == 0 and closes it when s & wmask == wmask (or s is the last)
     const int wmask = (1 << (log2g - 4)) - 1;
@@ -522,8 +625,8 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
       constexpr int kKind = decltype(kind)::value;
       constexpr bool kWin = decltype(win)::value;  // the matrix takes scale windows
       auto sq = [&](int q) { return kWin ? (q & (kDecodeWinGroups - 1)) ^ qx : q; };
-      if (s > 0 && !lanes_wait(full_bar(slot), parity, status)) return false;
-      if (kWin && (s & wmask) == 0) {
+      if (s > s0 && !lanes_wait(full_bar(slot), parity, status)) return false;
+      if (kWin && (s == s0 || (s & wmask) == 0)) {
         const int ub = units_u & 1;
         if (!lanes_wait(sfull_bar(ub), (units_u >> 1) & 1, status)) return false;
         ubase = reinterpret_cast<const float*>(ubuf + ub * ub_bytes);
@@ -656,7 +759,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(empty_bar(slot));
-      if (kWin && ((s & wmask) == wmask || s + 1 == nseg)) {
+      if (kWin && ((s & wmask) == wmask || s + 1 == s1)) {
         if (lane == 0) mbar_arrive(sempty_bar(units_u & 1));  // after the __syncwarp
         ++units_u;
       }
@@ -670,10 +773,12 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     auto run = [&](auto kind, auto win) {
       if constexpr (kTwoTiles) {
         // (two n-tiles: no register room for a second chunk body)
-        for (int s = 0; s < nseg && ok; ++s) ok = segment(s, std::true_type{}, kind, win);
+        for (int s = s0; s < s1 && ok; ++s) ok = segment(s, std::true_type{}, kind, win);
       } else {
-        for (int s = 0; s < nfull && ok; ++s) ok = segment(s, std::false_type{}, kind, win);
-        if (ok && nfull < nseg) ok = segment(nfull, std::true_type{}, kind, win);
+        // the segments inside k, then the one reaching past k if this piece has it
+        const int e = s1 < nfull ? s1 : nfull;
+        for (int s = s0; s < e && ok; ++s) ok = segment(s, std::false_type{}, kind, win);
+        if (ok && s1 > nfull) ok = segment(nfull, std::true_type{}, kind, win);
       }
     };
     auto run_kind = [&](auto kind) {
@@ -718,6 +823,57 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
         if (lane == 0) mbar_arrive(rempty_bar(wr, pb));
       }
       ++units_r;
+    }
+    if (kh == 0 && pieces > 1) {
+      // Pieces of k: CTA q > 0 of the cluster stores its partial sums of this row
+      // warp into the first CTA's shared memory (st.async, each store completing its
+      // bytes on the first CTA's "received" barrier of the row warp) and keeps its
+      // shared memory until the first CTA has them all; the first CTA adds them in
+      // piece order after its own piece 0 (the same sums in the same order whatever
+      // the timing) and stores the outputs.
+      constexpr int kLane = xpart_lane_floats<kTwoTiles>();
+      const uint32_t rank = cluster_rank();
+      cluster_wait();
+      // only the lanes holding tokens below m (tokens 2t, 2t + 1 and 8 + 2t, 9 + 2t)
+      const bool v0 = 2 * t < m, v1 = kTwoTiles && 8 + 2 * t < m;
+      if (rank != 0) {
+        const uint32_t dst = map_to_rank(
+            smem_u32(xpart + (((rank - 1) * kRowWarps + wr) * 32 + lane) * kLane), 0);
+        const uint32_t bar = map_to_rank(xfull_bar(wr), 0);
+#pragma unroll
+        for (int r = 0; r < kTiles; ++r) {
+          if (v0) st_async_f4(dst + 16 * r, make_float4(acc[r][0], acc[r][1], acc[r][2], acc[r][3]), bar);
+          if (v1)
+            st_async_f4(dst + 16 * (2 + r), make_float4(acc1[r][0], acc1[r][1], acc1[r][2], acc1[r][3]),
+                        bar);
+        }
+        if (!lanes_wait(xdone_bar(wr), 0, status)) return;
+        continue;  // (the end of the stream follows)
+      }
+      if (!lanes_wait_cluster(xfull_bar(wr), 0, status)) return;
+      // every piece has landed: the other CTAs may leave (nothing to release)
+      if (lane + 1 < pieces) mbar_arrive_remote_signal(map_to_rank(xdone_bar(wr), lane + 1));
+      for (int q = 1; q < pieces; ++q) {
+        const float4* v = reinterpret_cast<const float4*>(
+            xpart + (((q - 1) * kRowWarps + wr) * 32 + lane) * kLane);
+#pragma unroll
+        for (int r = 0; r < kTiles; ++r) {
+          if (v0) {
+            const float4 a0 = v[r];
+            acc[r][0] += a0.x;
+            acc[r][1] += a0.y;
+            acc[r][2] += a0.z;
+            acc[r][3] += a0.w;
+          }
+          if (v1) {
+            const float4 a1 = v[2 + r];
+            acc1[r][0] += a1.x;
+            acc1[r][1] += a1.y;
+            acc1[r][2] += a1.z;
+            acc1[r][3] += a1.w;
+          }
+        }
+      }
     }
     if (kh == 0) {
       // C fragment of tile r: rows rl + 16r (slots 0, 1) and + 8 (2, 3), tokens 2t, 2t + 1
@@ -773,6 +929,45 @@ uint32_t* dsched_base() {
 
 }  // namespace
 
+// Clusters of p CTAs of `kernel` (at `smem` bytes of shared memory each) that can
+// be resident at once, asked of the runtime once per kernel, size and device.
+template <typename K>
+cudaError_t max_active_clusters(K* kernel, int p, int smem, int threads, int* out) {
+  struct Entry {
+    const void* kernel;
+    int p, smem, dev, n;
+  };
+  static std::mutex mu;
+  static Entry cache[64];
+  static int used = 0;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const void* key = reinterpret_cast<const void*>(kernel);
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < used; ++i)
+    if (cache[i].kernel == key && cache[i].p == p && cache[i].smem == smem && cache[i].dev == dev) {
+      *out = cache[i].n;
+      return cudaSuccess;
+    }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(p), 1, 1);
+  cfg.blockDim = dim3(static_cast<unsigned>(threads), 1, 1);
+  cfg.dynamicSmemBytes = static_cast<size_t>(smem);
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(p);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if ((e = cudaOccupancyMaxActiveClusters(&n, kernel, &cfg)) != cudaSuccess) return e;
+  if (used < 64) cache[used++] = Entry{key, p, smem, dev, n};
+  *out = n;
+  return cudaSuccess;
+}
+
 cudaError_t launch_decode(DecodeBatch& b, int num_sms, cudaStream_t stream) {
   static std::atomic<uint32_t> seq{0};
   // longest rows first: the units claimed last are the shortest (matrices and
@@ -794,15 +989,18 @@ cudaError_t launch_decode(DecodeBatch& b, int num_sms, cudaStream_t stream) {
       b.maps[d] = tmp.maps[d];
     }
   }
-  int64_t units = 0;
+  int64_t blocks_of_rows = 0;
+  int min_nseg = 1 << 30;
   for (int d = 0; d < b.count; ++d) {
-    b.mats[d].unit0 = static_cast<int32_t>(units);
-    units += (b.mats[d].n + kRows - 1) / kRows;
+    blocks_of_rows += (b.mats[d].n + kRows - 1) / kRows;
+    const int nseg = static_cast<int>((b.mats[d].k + kSegK - 1) / kSegK);
+    min_nseg = nseg < min_nseg ? nseg : min_nseg;
   }
-  if (units >= (int64_t{1} << 31)) return cudaErrorInvalidValue;
-  b.total_units = static_cast<int32_t>(units);
-  if (b.total_units <= 0) return cudaSuccess;
-  const int64_t blocks = units < num_sms ? units : num_sms;
+  if (blocks_of_rows >= (int64_t{1} << 28)) return cudaErrorInvalidValue;
+  if (blocks_of_rows <= 0) {
+    b.total_units = 0;
+    return cudaSuccess;
+  }
   // scale buffers: the largest unit of scales among unit-mode matrices, a window
   // (256 rows x 32 groups, 1024-byte aligned for the swizzle) if any matrix takes
   // windows; ring slot: codes + the widest per-segment scale area + x of the m tokens
@@ -825,22 +1023,74 @@ cudaError_t launch_decode(DecodeBatch& b, int num_sms, cudaStream_t stream) {
   b.scale_bytes = kRows * sgroups * 4;
   b.slot_bytes = (kCodeBytes + b.scale_bytes + b.m * kXTokBytes + 1023) & ~1023;
   const int red = b.m > 8 ? red_bytes<true>() : red_bytes<false>();
-  const int fit = (kSmemLimit - 1024 - kHeadBytes - red - 2 * b.ubuf_bytes) / b.slot_bytes;
-  b.stages = fit < kMaxStages ? fit : kMaxStages;
-  if (b.stages < 2) return cudaErrorInvalidValue;
-  const int smem = 1024 + kHeadBytes + red + 2 * b.ubuf_bytes + b.stages * b.slot_bytes;
+  auto smem_for = [&](int pieces, int* stages) {
+    const int fixed = 1024 + kHeadBytes + red + xpart_bytes(b.m > 8, pieces) + 2 * b.ubuf_bytes;
+    const int fit = (kSmemLimit - fixed) / b.slot_bytes;
+    *stages = fit < kMaxStages ? fit : kMaxStages;
+    return fixed + *stages * b.slot_bytes;
+  };
   uint32_t* sched = dsched_base();
   if (sched == nullptr) return cudaErrorInvalidSymbol;
   sched += 2 * (seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
-  cudaError_t e;
   auto go = [&](auto two, auto f16) -> cudaError_t {
     constexpr bool kTwo = decltype(two)::value, kF16 = decltype(f16)::value;
-    cudaError_t err = ensure_smem_limit<decode_kernel<kTwo, kF16>>(kSmemLimit);
+    auto* kernel = decode_kernel<kTwo, kF16, false>;
+    auto* kernel_pieces = decode_kernel<kTwo, kF16, true>;
+    cudaError_t err = ensure_smem_limit<decode_kernel<kTwo, kF16, false>>(kSmemLimit);
     if (err != cudaSuccess) return err;
-    decode_kernel<kTwo, kF16><<<static_cast<unsigned>(blocks), DecodeCfg<kTwo>::kThreads, smem,
-                                stream>>>(b, sched);
-    return cudaSuccess;
+    // Pieces of k when the blocks of rows leave SMs idle: clusters of P CTAs
+    // (P = 8, 4 or 2, at most every matrix's segment count), the largest P whose
+    // clusters for all the blocks are resident at once.
+    int pieces = 1;
+    if (blocks_of_rows < num_sms) {
+      for (int p = 8; p >= 2; p >>= 1) {
+        int st = 0;
+        const int sm = smem_for(p, &st);
+        if (p > min_nseg || st < 2 || blocks_of_rows * p > num_sms) continue;
+        int nclusters = 0;
+        if ((err = ensure_smem_limit<decode_kernel<kTwo, kF16, true>>(kSmemLimit)) != cudaSuccess)
+          return err;
+        if (max_active_clusters(kernel_pieces, p, sm, DecodeCfg<kTwo>::kThreads, &nclusters) ==
+                cudaSuccess &&
+            nclusters >= blocks_of_rows) {
+          pieces = p;
+          break;
+        }
+      }
+    }
+    b.pieces = pieces;
+    int64_t units = 0;
+    for (int d = 0; d < b.count; ++d) {
+      b.mats[d].unit0 = static_cast<int32_t>(units);
+      units += ((b.mats[d].n + kRows - 1) / kRows) * pieces;
+    }
+    b.total_units = static_cast<int32_t>(units);
+    int stages = 0;
+    const int smem = smem_for(pieces, &stages);
+    b.stages = stages;
+    if (b.stages < 2) return cudaErrorInvalidValue;
+    if (pieces == 1) {
+      // persistent: one CTA per SM at most, units claimed from the scheduler
+      const int64_t blocks = units < num_sms ? units : num_sms;
+      kernel<<<static_cast<unsigned>(blocks), DecodeCfg<kTwo>::kThreads, smem, stream>>>(b, sched);
+      return cudaSuccess;
+    }
+    // one CTA per unit, clusters of `pieces` CTAs over one block of rows
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(units), 1, 1);
+    cfg.blockDim = dim3(DecodeCfg<kTwo>::kThreads, 1, 1);
+    cfg.dynamicSmemBytes = static_cast<size_t>(smem);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = static_cast<unsigned>(pieces);
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel_pieces, b, sched);
   };
+  cudaError_t e;
   if (b.m > 8)
     e = b.in_f16 ? go(std::true_type{}, std::true_type{}) : go(std::true_type{}, std::false_type{});
   else

@@ -45,6 +45,10 @@ struct DecodeBatch {
   int32_t stages;         // ring slots
   int32_t ubuf_bytes;     // one unit- or window-scale buffer (two are kept)
   int32_t in_f16;         // 1: fp16 activations in every matrix (else bf16)
+  // pieces of k per block of rows (set by the launcher): 1, a persistent grid
+  // claiming units; P > 1, clusters of P CTAs, CTA p of a cluster taking piece p
+  // of one block's segments, the first CTA adding the others' partial sums
+  int32_t pieces;
 };
 
 // Reorders b.mats / b.maps (decreasing k) and sets unit0 and total_units.

@@ -500,6 +500,52 @@ def test_batched_decode_scale_modes_past_the_map_limit(tq):
                     max_rel_rms=3e-2 if it["y"].dtype == torch.bfloat16 else 2e-2)
 
 
+# A launch with fewer 256-row blocks than SMs cuts k into P pieces (clusters of P
+# CTAs, the first adding the others' partial sums): one matrix per call here, each
+# scale mode, ragged k and rows, pieces that end inside a window of scales.
+_SPLIT_SHAPES = [
+    (8512, 2048, 128),   # Mamba-2 1.3B in_proj: 34 blocks, unit scales
+    (2048, 4096, 128),   # out_proj: 8 blocks
+    (520, 1088, 64),     # k/g = 17: per-segment scales; 3 segments, the last ragged
+    (264, 4608, 128),    # k/g = 36: scale windows cut by the pieces
+    (300, 18432, 512),   # k/g = 36 at g = 512, 36 segments
+    (136, 2560, 32),     # k/g = 80 windows of 32 groups at g = 32
+]
+
+
+@pytest.mark.parametrize("n,k,g", _SPLIT_SHAPES)
+@pytest.mark.parametrize("m", [1, 5, 8, 9, 16])
+def test_decode_pieces_of_k(tq, n, k, g, m):
+    w, x, dy, w_hat, codes, s = _setup(tq, n, k, m, g, seed=n + k + m)
+    xd = x.cuda()
+    y = tq.linear_fwd(xd, codes, s, g)
+    yb = tq.linear_fwd(xd, codes, s, g, out_dtype=torch.bfloat16)
+    y2 = tq.linear_fwd(xd, codes, s, g)
+    tq.device_status()
+    check_close(to_np(y), O.linear_fwd(x, w_hat), f"Y pieces n={n} k={k} g={g} m={m}")
+    assert torch.equal(y, y2)                      # the same sums in the same order
+    assert torch.equal(yb, y.to(torch.bfloat16))
+
+
+def test_decode_persistent_160_blocks(tq):
+    """A batch of 160 blocks of rows (no pieces: a persistent grid claiming units),
+    compared in full."""
+    g, m = 128, 6
+    items = []
+    for i in range(40):
+        n, k = 1024 - 8 * (i % 3), 1024 + 512 * (i % 2)
+        w = synth.latent_weights(n, k, seed=5000 + i)
+        x = synth.activations_bf16(m, k, seed=5000 + i)
+        codes, s, z = _quant(tq, w, g)
+        items.append(dict(x=x.cuda(), codes=codes, scales=s, g=g,
+                          y=torch.empty((m, n), device="cuda"),
+                          ref=O.linear_fwd(x, validated_w_hat(w, g, codes, s, z))))
+    tq.linear_fwd_batched(items, m)
+    tq.device_status()
+    for i, it in enumerate(items):
+        check_close(it["y"], it["ref"], f"persistent Y[{i}]")
+
+
 def test_prefill_few_rows_many_tokens(tq):
     """64 weight rows (half a tile) against 40000 tokens (157 token tiles with a
     ragged last one), all three products."""
