@@ -441,10 +441,8 @@ def time_e2e(p: Prefill, steps, warmup):
     return ms, h2d, d2h
 
 
-def decode_sweep(tq, m_list, steps, warmup):
-    """Decode forward over all 48 layers' packed in_proj and out_proj (one batched call)."""
-    gen = torch.Generator(device="cuda")
-    gen.manual_seed(1234)
+def _decode_mats(tq, gen):
+    """The packed in_proj and out_proj of all 48 layers, layer by layer."""
     mats = []
     for layer in range(N_LAYERS):
         for (n, k) in (IN_PROJ, OUT_PROJ):
@@ -452,6 +450,14 @@ def decode_sweep(tq, m_list, steps, warmup):
             codes, s, _ = tq.quantize(w, G)
             mats.append((n, k, codes, s))
             del w
+    return mats
+
+
+def decode_sweep(tq, m_list, steps, warmup):
+    """Decode forward over all 48 layers' packed in_proj and out_proj (one batched call)."""
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(1234)
+    mats = _decode_mats(tq, gen)
     out = {}
     for m in m_list:
         items = []
@@ -475,6 +481,53 @@ def decode_sweep(tq, m_list, steps, warmup):
                      it["y"].numel() * 4 for it in items)
         out[f"M={m}"] = {"us": round(ms * 1e3, 2), "GB/s": round(nbytes / ms / 1e6, 1),
                          "bytes": nbytes}
+    tq.device_status()
+    return out
+
+
+def decode_per_layer(tq, m_list, replays, warmup):
+    """One decode step as a model runs it: layer after layer, in_proj then out_proj,
+    one tq_linear_fwd launch each (96 launches in stream order), captured once in a
+    CUDA graph and replayed, so that the host's per-call cost stays out of the
+    device time. The 351 MB of codes exceed L2: every replay streams them from HBM."""
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(4321)
+    mats = _decode_mats(tq, gen)
+    out = {}
+    for m in m_list:
+        calls = []
+        for (n, k, codes, s) in mats:
+            x = torch.randn((m, k), generator=gen, device="cuda").to(torch.bfloat16)
+            calls.append((x, codes, s, torch.empty((m, n), device="cuda")))
+        stream = torch.cuda.Stream()
+        stream.wait_stream(torch.cuda.current_stream())
+
+        def step():
+            for (x, codes, s, y) in calls:
+                tq.linear_fwd(x, codes, s, G, y=y, stream=stream)
+
+        with torch.cuda.stream(stream):
+            step()  # outside the capture: attributes, tensor maps, cluster sizes
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            step()
+        for _ in range(warmup):
+            graph.replay()
+        torch.cuda.synchronize()
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record()
+        for _ in range(replays):
+            graph.replay()
+        t1.record()
+        torch.cuda.synchronize()
+        us = t0.elapsed_time(t1) * 1e3 / replays
+        nbytes = sum(c.numel() * 4 + s_.numel() * 4 + x.numel() * 2 + y.numel() * 4
+                     for (x, c, s_, y) in calls)
+        out[f"M={m}"] = {"us_per_step": round(us, 1), "us_per_layer": round(us / N_LAYERS, 2),
+                         "launches": len(calls), "GB/s": round(nbytes / us / 1e3, 1)}
+        del graph
     tq.device_status()
     return out
 
@@ -986,6 +1039,7 @@ def main():
     if not args.no_extra and rank == 0:
         line["extra"] = {
             "decode_48_layers": decode_sweep(tq, (1, 4, 16), 20, 3),
+            "decode_48_layers_launch_per_projection": decode_per_layer(tq, (1, 4, 16), 20, 3),
             "quantize_48_layers_g128": quantize_sweep(tq, 5, 2),
             "out_proj_step": out_proj_step(tq, 200, 10),
             "in_proj_step_fp16_activations": out_proj_step(tq, 200, 10, IN_PROJ, torch.float16),

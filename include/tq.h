@@ -296,7 +296,11 @@ TQ_API tq_status tq_linear_fwd(const void* x, int64_t m, int64_t k,
  *   dW launches of one device share the library's 40 MB workspace (the partial
  *   sums of the tiles split across SMs): each dW launch waits for the device's
  *   previous dW launch, on whatever stream either was issued (an event the
- *   library records after every dW launch, waited on by the next one).
+ *   library records after every dW launch, waited on by the next one). A call
+ *   made while `stream` is being captured into a CUDA graph takes no part in
+ *   that: the graph's own dependencies order its dW nodes, so a graph must not
+ *   leave two dW nodes unordered, nor be replayed beside a dW launch on another
+ *   stream.
  */
 TQ_API tq_status tq_linear_bwd(const void* dy, const void* x, int64_t m, int64_t n, int64_t k,
                         const uint32_t* codes, const uint32_t* codes_t, const float* scales,

@@ -483,11 +483,19 @@ cudaError_t launch_dw_gemm(const CUtensorMap& tmap_x, const CUtensorMap& tmap_dy
   // The stream-K workspace and counters are shared by the device's dW launches:
   // every launch after the first waits for the previous one, whatever stream
   // either was issued on (a wait on the same stream's own last event costs
-  // nothing on the device).
+  // nothing on the device). A launch captured into a CUDA graph may not depend on
+  // work outside the capture: there the graph's own edges order the dW nodes, and
+  // the event is neither waited on nor recorded.
   std::lock_guard<std::mutex> lock(g_dw_order_mu);
   int dev = 0;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
   if (dev >= kOrderDevices) return cudaErrorInvalidDevice;
+  cudaStreamCaptureStatus capture = cudaStreamCaptureStatusNone;
+  if ((e = cudaStreamIsCapturing(stream, &capture)) != cudaSuccess) return e;
+  if (capture != cudaStreamCaptureStatusNone) {
+    dw_gemm_kernel<<<static_cast<unsigned>(2 * pairs), kThreads, smem, stream>>>(tmap_x, tmap_dy, a);
+    return cudaGetLastError();
+  }
   if (g_dw_done[dev] == nullptr &&
       (e = cudaEventCreateWithFlags(&g_dw_done[dev], cudaEventDisableTiming)) != cudaSuccess)
     return e;
