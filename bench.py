@@ -920,6 +920,19 @@ def run_only(args):
         res = decode_sweep(tq, (1,), args.steps, args.warmup)
         print(json.dumps({"only": "decode", **res}), flush=True)
         return
+    if args.only == "decode_single":
+        # one in_proj projection at one token, one launch per call (k cut into pieces)
+        n, k = IN_PROJ
+        w = torch.randn((n, k), device="cuda") * 0.02
+        codes, s, _ = tq.quantize(w, G)
+        x = torch.randn((1, k), device="cuda").to(torch.bfloat16)
+        y = torch.empty((1, n), device="cuda")
+        for _ in range(args.warmup + args.steps):
+            tq.linear_fwd(x, codes, s, G, y=y)
+        torch.cuda.synchronize()
+        tq.device_status()
+        print(json.dumps({"only": "decode_single", "n": n, "k": k, "m": 1}), flush=True)
+        return
     if args.only == "adamw":
         n, k = IN_PROJ
         w = torch.randn((n, k), device="cuda") * 0.02
@@ -978,7 +991,8 @@ def main():
     ap.add_argument("--impl", default="tq", choices=["tq", "reference"])
     ap.add_argument("--no-extra", action="store_true", help="skip decode/quantize sweeps")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
-    ap.add_argument("--only", choices=["quantize", "quantize_t", "transpose", "fwd", "dx", "dw", "decode", "adamw",
+    ap.add_argument("--only", choices=["quantize", "quantize_t", "transpose", "fwd", "dx", "dw", "decode",
+                                       "decode_single", "adamw",
                                        "given", "scale_grad", "alpha_grad"],
                     help="profiling aid: run just this kernel of the step (or the batched "
                          "M=1 decode) --warmup + --steps times and print its time")
