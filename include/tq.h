@@ -275,6 +275,10 @@ TQ_API tq_status tq_adamw(float* p, const float* grad, float* m, float* v, int64
  *   pieces run by one thread-block cluster whose first CTA adds the others'
  *   partial sums to its own in piece order: the same result on every run (its
  *   rounding differs from that of an uncut launch by the order of the sums).
+ *   Decode launches use programmatic dependent launch: one may start its CTAs
+ *   while the previous kernel on the stream is still running, but before that
+ *   kernel has completed it only prefetches codes and scales into L2 (coherent
+ *   with any write still to come); every other read and every write waits.
  */
 TQ_API tq_status tq_linear_fwd(const void* x, int64_t m, int64_t k,
                         const uint32_t* codes, const float* scales, int64_t n, int32_t g,

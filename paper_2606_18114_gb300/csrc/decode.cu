@@ -293,6 +293,28 @@ __device__ __forceinline__ void st_async_f4(uint32_t cluster_addr, float4 v, uin
       : "memory");
 }
 
+// Programmatic dependent launch. launch_dependents lets the next launch on the stream
+// (one made with the programmatic-serialisation attribute) start its CTAs on SMs
+// that this grid leaves free; wait holds this thread until the previous grid on
+// the stream has completed and its writes are visible.
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// L2 prefetches (no shared memory written, no barrier): L2 is where the device's
+// writes meet, so a line fetched before the previous grid has finished writing it
+// is updated in place and later loads see the new data.
+__device__ __forceinline__ void prefetch_l2_tile(const CUtensorMap* map, int32_t x, int32_t y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y)
+               : "memory");
+}
+__device__ __forceinline__ void prefetch_l2(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 // Binary search: matrix d with unit0[d] <= u < unit0[d + 1].
 __device__ __forceinline__ int find_mat(const DecodeBatch& b, int u) {
   int lo = 0, hi = b.count - 1;
@@ -375,6 +397,9 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
   // barrier completes: arrive now, wait only before the first access to another
   // CTA's shared memory (long since complete by then).
   if (pieces > 1) cluster_arrive();
+  // the next decode launch on the stream may start its CTAs on the SMs this grid
+  // leaves free; they prefetch into L2 and then wait for this grid (pdl_wait)
+  pdl_launch_dependents();
 
   if (warp == kConsumers) {
     // ------------------------------------------------------------ producer
@@ -386,6 +411,29 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
     int units_u = 0;  // units and windows whose scales went through the buffers
     bool ok = true;
     int claims = 0;
+    if (lane == 0 && static_cast<int>(blockIdx.x) < b.total_units) {
+      // Before the previous grid on the stream has finished: bring this CTA's first
+      // unit's codes (as many segments as the ring holds) and scales into L2.
+      const int u = static_cast<int>(blockIdx.x);
+      const int d = find_mat(b, u);
+      const DecodeMat& mt = b.mats[d];
+      const int nseg = static_cast<int>((mt.k + kSegK - 1) / kSegK);
+      const int local = u - mt.unit0;
+      const int piece = local % pieces;
+      const int64_t row0 = static_cast<int64_t>(local / pieces) * kRows;
+      const int s0 = piece * nseg / pieces, s1 = (piece + 1) * nseg / pieces;
+      for (int s = s0; s < s1 && s < s0 + stages; ++s)
+        prefetch_l2_tile(&b.maps[d], s * (kSegK / 16), static_cast<int32_t>(row0));
+      const int64_t gpr = mt.k >> mt.log2g;
+      if (mt.scale_mode == kDecodeScaleUnit) {
+        const int64_t rows = mt.n - row0 < kRows ? mt.n - row0 : kRows;
+        prefetch_l2(mt.scales + row0 * gpr, static_cast<uint32_t>(rows * gpr * 4));
+      } else if (mt.scale_mode == kDecodeScaleWin) {
+        prefetch_l2_tile(&b.maps[mt.smap], (s0 >> (mt.log2g - 4)) * kDecodeWinGroups,
+                         static_cast<int32_t>(row0));
+      }
+    }
+    pdl_wait();  // nothing of the previous grid's output is read or overwritten before
     for (;;) {
       // the first unit of every CTA is dealt (blocks <= units), later ones claimed
       // (with pieces of k every CTA takes its one dealt unit)
@@ -530,6 +578,7 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
   }
 
   // -------------------------------------------------------------- consumers
+  pdl_wait();  // (their outputs may be read by the previous grid until it completes)
   // Warp w owns rows 32wr .. 32wr + 31 of the unit (wr = w % 8) as two m16 tiles
   // that share every activation fragment, over the chunks c of each segment with
   // c / (4 / kSplit) == w / 8; lane (g, t) holds rows 32wr + 16r + g (+8) of tile r.
@@ -1069,25 +1118,30 @@ cudaError_t launch_decode(DecodeBatch& b, int num_sms, cudaStream_t stream) {
     const int smem = smem_for(pieces, &stages);
     b.stages = stages;
     if (b.stages < 2) return cudaErrorInvalidValue;
-    if (pieces == 1) {
-      // persistent: one CTA per SM at most, units claimed from the scheduler
-      const int64_t blocks = units < num_sms ? units : num_sms;
-      kernel<<<static_cast<unsigned>(blocks), DecodeCfg<kTwo>::kThreads, smem, stream>>>(b, sched);
-      return cudaSuccess;
-    }
-    // one CTA per unit, clusters of `pieces` CTAs over one block of rows
+    // Every decode launch may start before the previous launch on the stream has
+    // completed (programmatic serialisation): its CTAs set up and prefetch into L2,
+    // then wait for that grid before reading or writing anything it might touch.
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(static_cast<unsigned>(units), 1, 1);
     cfg.blockDim = dim3(DecodeCfg<kTwo>::kThreads, 1, 1);
     cfg.dynamicSmemBytes = static_cast<size_t>(smem);
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = static_cast<unsigned>(pieces);
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    if (pieces == 1) {
+      // persistent: one CTA per SM at most, units claimed from the scheduler
+      cfg.gridDim = dim3(static_cast<unsigned>(units < num_sms ? units : num_sms), 1, 1);
+      cfg.numAttrs = 1;
+      return cudaLaunchKernelEx(&cfg, kernel, b, sched);
+    }
+    // one CTA per unit, clusters of `pieces` CTAs over one block of rows
+    cfg.gridDim = dim3(static_cast<unsigned>(units), 1, 1);
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = static_cast<unsigned>(pieces);
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, kernel_pieces, b, sched);
   };
   cudaError_t e;
