@@ -44,6 +44,8 @@ constexpr int kExpWarp0 = 6;                 // warps 6..13: two expansion warpg
 constexpr int kThreads = 14 * 32;
 constexpr int kKBlock = 128;                 // reduction elements per stage
 constexpr int kCodesBytes = 4096;            // 128 rows x 8 code words
+// dX with at most this many k-blocks per tile (n <= 4096) runs the ping-pong layout
+constexpr int kDxPingPongMaxKb = 32;
 
 // Rings: kSmem shared-memory stages (activation tile as two 64-wide swizzled halves
 // + codes, filled by TMA) and kAStages tensor-memory stages of expanded weights
@@ -66,14 +68,17 @@ constexpr int kCodesBytes = 4096;            // 128 rows x 8 code words
 //     stream (~66 B per cycle into each SM) instead of pausing it. A deep A ring
 //     hides the commit -> expansion -> MMA round trip: two A stages beside a ring of
 //     three 128-token accumulator halves ran the forward in 0.411 ms;
-//   dX, 256 tokens: one accumulator and four A stages in a ring over the launch (its
-//     tiles are 67 k-blocks long at in_proj, so the drain is a small share; the
-//     ping-pong layout ran it 1 % slower);
+//   dX, 256 tokens: with more than kDxPingPongMaxKb k-blocks per tile, one
+//     accumulator and four A stages in a ring over the launch (its tiles are 67
+//     k-blocks long at in_proj, so the drain is a small share: the ping-pong layout
+//     ran it 1.6 % slower); with fewer, ping-pong as the forward (out_proj, 16
+//     k-blocks: 0.210 -> 0.201 ms; equal at 32 and 48);
 //   16 tokens: two accumulators and four A stages.
-template <int MODE, int BN>
+template <int MODE, int BN, bool PP>
 struct TsLayout {
   static_assert(BN == 16 || BN == 256, "tile tokens");
-  static constexpr bool kPingPong = BN == 256 && MODE == kTsFwd;
+  static_assert(!PP || BN == 256, "ping-pong: two 256-column halves");
+  static constexpr bool kPingPong = PP;
   static constexpr int kSmem = BN == 16 ? 16 : 3;
   static constexpr int kAStages = 4;
   static constexpr int kAcc = BN == 256 ? 1 : 2;
@@ -130,11 +135,11 @@ __device__ __forceinline__ void expand_word(uint32_t w, uint32_t hs, uint32_t* a
   for (int j = 0; j < 8; ++j) a[j] = bmul2<F16>((w << (14 - 2 * j)) & 0xC000C000u, hs);
 }
 
-template <int MODE, int BN, bool F16>
+template <int MODE, int BN, bool F16, bool PP>
 __global__ void __launch_bounds__(kThreads, 1)
     ts_gemm_kernel(const __grid_constant__ CUtensorMap tmap_b,
                    const __grid_constant__ CUtensorMap tmap_codes, const TsArgs args) {
-  using L = TsLayout<MODE, BN>;
+  using L = TsLayout<MODE, BN, PP>;
   constexpr int kSmem = L::kSmem, kAS = L::kAStages, kAcc = L::kAcc;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align_shared<1024>(smem_raw);
@@ -576,16 +581,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int MODE, int BN, bool F16>
+template <int MODE, int BN, bool F16, bool PP>
 cudaError_t launch_impl(const CUtensorMap& tb, const CUtensorMap& tc, const TsArgs& a,
                         int num_sms, cudaStream_t stream) {
-  using L = TsLayout<MODE, BN>;
+  using L = TsLayout<MODE, BN, PP>;
   // Enough shared memory that two CTAs never share an SM (each holds up to 512
   // tensor-memory columns).
   size_t smem = L::kBytes + 1024;
   if (smem < 116 * 1024) smem = 116 * 1024;
-  auto kern = ts_gemm_kernel<MODE, BN, F16>;
-  cudaError_t e = ensure_smem_limit<ts_gemm_kernel<MODE, BN, F16>>(static_cast<int>(smem));
+  auto kern = ts_gemm_kernel<MODE, BN, F16, PP>;
+  cudaError_t e = ensure_smem_limit<ts_gemm_kernel<MODE, BN, F16, PP>>(static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   const int64_t rows = MODE == kTsFwd ? a.wn : a.wk;
   const int64_t tiles = ((rows + 127) / 128) * ((a.m + BN - 1) / BN);
@@ -602,14 +607,21 @@ namespace {
 template <bool F16>
 cudaError_t launch_typed(int mode, int bn, const CUtensorMap& tb, const CUtensorMap& tc,
                          const TsArgs& a, int num_sms, cudaStream_t stream) {
+  // dX tiles reduce over n: with few k-blocks per tile the drain of the single
+  // accumulator is a large share of each tile, so short reductions take ping-pong
+  const bool dx_pp = (a.wn + kKBlock - 1) / kKBlock <= kDxPingPongMaxKb;
   if (mode == kTsFwd) {
-    if (bn == 256) return launch_impl<kTsFwd, 256, F16>(tb, tc, a, num_sms, stream);
+    if (bn == 256) return launch_impl<kTsFwd, 256, F16, true>(tb, tc, a, num_sms, stream);
   } else if (mode == kTsDx) {
-    if (bn == 16) return launch_impl<kTsDx, 16, F16>(tb, tc, a, num_sms, stream);
-    if (bn == 256) return launch_impl<kTsDx, 256, F16>(tb, tc, a, num_sms, stream);
+    if (bn == 16) return launch_impl<kTsDx, 16, F16, false>(tb, tc, a, num_sms, stream);
+    if (bn == 256)
+      return dx_pp ? launch_impl<kTsDx, 256, F16, true>(tb, tc, a, num_sms, stream)
+                   : launch_impl<kTsDx, 256, F16, false>(tb, tc, a, num_sms, stream);
   } else if (mode == kTsDxT) {
-    if (bn == 16) return launch_impl<kTsDxT, 16, F16>(tb, tc, a, num_sms, stream);
-    if (bn == 256) return launch_impl<kTsDxT, 256, F16>(tb, tc, a, num_sms, stream);
+    if (bn == 16) return launch_impl<kTsDxT, 16, F16, false>(tb, tc, a, num_sms, stream);
+    if (bn == 256)
+      return dx_pp ? launch_impl<kTsDxT, 256, F16, true>(tb, tc, a, num_sms, stream)
+                   : launch_impl<kTsDxT, 256, F16, false>(tb, tc, a, num_sms, stream);
   }
   return cudaErrorInvalidValue;
 }
