@@ -35,11 +35,24 @@
 // weights as the 16 x 16 A operand and up to 8 tokens as the n8 B operand (two B
 // tiles for 9..16 tokens). The reduction index of the MMA is permuted identically on both
 // operands so that lane (g, t) (g = lane / 4, t = lane % 4) consumes exactly code
-// words 2t, 2t+1 of the chunk for rows g and g + 8 and the contiguous 64 bytes
-// x[token g][32t .. 32t + 31]: MMA kb takes offsets 32t + 4kb + {0,1} for
-// fragment slots (2t, 2t+1) and 32t + 4kb + {2,3} for slots (2t+8, 2t+9). Tokens
-// past m read token m - 1: their output columns are never stored, and MMA
-// columns do not mix.
+// words t and t + 4 of the chunk (k offsets 16t .. 16t + 15 and 64 + 16t .. 64 + 16t
+// + 15) for rows g and g + 8, and x[token g] at the same offsets: MMA kb takes word
+// w = t (kb < 4) or t + 4 (kb >= 4), offsets 16w + 4 (kb % 4) + {0,1} for fragment
+// slots (2t, 2t+1) and + {2,3} for slots (2t+8, 2t+9). Tokens past m read token
+// m - 1: their output columns are never stored, and MMA columns do not mix.
+//
+// Pieces of k: a launch with fewer blocks of 256 rows than SMs (one layer's
+// projection at a time) runs clusters of P = 8, 4 or 2 CTAs instead of the
+// persistent grid, one cluster per block, CTA p streaming segments [p nseg / P,
+// (p + 1) nseg / P); the other CTAs send their fp32 partial sums (the lanes that
+// hold tokens below m) into the first CTA's shared memory with st.async, counted on
+// its barrier, and the first CTA adds them to its own in piece order before the
+// store — the same sums in the same order on every run.
+//
+// Every launch is a programmatic dependent launch: its CTAs may start on SMs the
+// previous grid on the stream leaves free, set up, prefetch their first unit's
+// codes and scales into L2 (coherent with any write still to come), and then wait
+// for that grid before any other global access.
 //
 // Expansion: pair j of a code word -> bf16x2 (2c, 2c) by ((w << (14 - 2j)) &
 // 0xC000C000) (layout of include/tq.h). For g >= 128 a chunk lies in one group:
