@@ -1,7 +1,8 @@
 """GB300-native grouped ternary (W1.58A16) linear layer.
 
 ``tq`` is the ctypes binding of libtq (include/tq.h); ``ternary_linear`` wraps it as a
-torch autograd function and module (TernaryLinear, §3.1); ``synth`` draws the seeded
+torch autograd function and module (TernaryLinear, §3.1) and its packed inference
+form (PackedTernaryLinear); ``synth`` draws the seeded
 synthetic inputs; ``build`` compiles libtq.so for sm_103a.
 """
 from . import synth  # noqa: F401

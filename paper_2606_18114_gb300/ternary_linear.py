@@ -9,8 +9,10 @@ runs in libtq's kernels (``tq.quantize_with_transpose``, ``tq.linear_fwd``,
 none).
 
 Shapes: ``x [..., in_features]`` (bf16 or fp16, last dimension contiguous after a
-reshape), ``weight [out_features, in_features]`` fp32; in_features a multiple of 16 and of
+reshape), ``weight [out_features, in_features]`` fp32; in_features a multiple of 64 and of
 the group size g, out_features a multiple of 8 (the backward kernels' requirement).
+``PackedTernaryLinear`` (from ``TernaryLinear.pack()``) is the inference form: only the
+2-bit codes and group scales, no latent weights, no gradient.
 """
 from __future__ import annotations
 
@@ -75,8 +77,8 @@ class TernaryLinear(torch.nn.Module):
     def __init__(self, in_features: int, out_features: int, g: int = 128, out_dtype=None,
                  device="cuda", init_std: float = 0.02):
         super().__init__()
-        if in_features % 16 or in_features % g:
-            raise ValueError("in_features must be a multiple of 16 and of g")
+        if in_features % 64 or in_features % g:
+            raise ValueError("in_features must be a multiple of 64 and of g")
         if out_features % 8:
             raise ValueError("out_features must be a multiple of 8")
         self.in_features, self.out_features, self.g, self.out_dtype = (
@@ -94,6 +96,53 @@ class TernaryLinear(torch.nn.Module):
         if self._zeros is None:
             raise RuntimeError("no forward has run yet")
         return float(self._zeros.sum(dtype=torch.int64)) / self.weight.numel()
+
+    @torch.no_grad()
+    def pack(self) -> "PackedTernaryLinear":
+        """The inference form of the current weights: their 2-bit codes and group scales
+        (quantised once, here), without the fp32 latent weights."""
+        codes, scales, _ = tq.quantize(self.weight.detach().contiguous(), self.g)
+        return PackedTernaryLinear(codes, scales, self.in_features, self.g, self.out_dtype)
+
+    def extra_repr(self) -> str:
+        return f"in_features={self.in_features}, out_features={self.out_features}, g={self.g}"
+
+
+class PackedTernaryLinear(torch.nn.Module):
+    """Inference form of TernaryLinear (§8, storage): the weights held only as packed
+    ternary codes (uint32-as-int32 ``[out_features, in_features / 16]``, 16 codes per
+    word) and fp32 group scales ``[out_features, in_features / g]`` — 0.25 + 4/g bytes
+    per weight — and the forward y = x Ŵᵀ run on them: the decode kernel up to 16
+    tokens, the tensor-core GEMM beyond. No gradient flows through it."""
+
+    def __init__(self, codes: torch.Tensor, scales: torch.Tensor, in_features: int, g: int = 128,
+                 out_dtype=None):
+        super().__init__()
+        n = codes.shape[0]
+        if codes.dtype != torch.int32 or codes.shape != (n, in_features // 16):
+            raise ValueError("codes must be int32 [out_features, in_features / 16]")
+        if scales.dtype != torch.float32 or scales.shape != (n, in_features // g):
+            raise ValueError("scales must be fp32 [out_features, in_features / g]")
+        if in_features % 64 or in_features % g:
+            raise ValueError("in_features must be a multiple of 64 and of g")
+        if out_dtype is not None and out_dtype not in _OUT_TYPES:
+            raise TypeError(f"out_dtype must be fp32 or bf16, not {out_dtype}")
+        self.in_features, self.out_features, self.g, self.out_dtype = in_features, n, g, out_dtype
+        self.register_buffer("codes", codes.contiguous())
+        self.register_buffer("scales", scales.contiguous())
+
+    @torch.no_grad()
+    def forward(self, x: torch.Tensor) -> torch.Tensor:
+        if x.dtype not in (torch.bfloat16, torch.float16):
+            raise TypeError(f"x must be bf16 or fp16, not {x.dtype}")
+        if x.shape[-1] != self.in_features:
+            raise ValueError(f"x has {x.shape[-1]} features, the layer {self.in_features}")
+        out_dtype = self.out_dtype
+        if out_dtype is None:
+            out_dtype = torch.bfloat16 if x.dtype == torch.bfloat16 else torch.float32
+        x2 = x.reshape(-1, self.in_features).contiguous()
+        y = tq.linear_fwd(x2, self.codes, self.scales, self.g, out_dtype=out_dtype)
+        return y.reshape(*x.shape[:-1], self.out_features)
 
     def extra_repr(self) -> str:
         return f"in_features={self.in_features}, out_features={self.out_features}, g={self.g}"

@@ -102,3 +102,23 @@ def test_module_step_and_zero_ratio(tq):
     opt.step()
     tq.device_status()
     assert not torch.equal(layer.weight.detach(), w0)
+
+
+@pytest.mark.parametrize("m", [3, 300])
+def test_packed_inference_equals_the_training_forward(tq, m):
+    """TernaryLinear.pack(): the codes and scales of the current weights, 2-bit
+    storage, the same forward kernels (decode up to 16 tokens, the GEMM beyond)."""
+    from paper_2606_18114_gb300.ternary_linear import PackedTernaryLinear, TernaryLinear
+    torch.manual_seed(m)
+    layer = TernaryLinear(1024, 520, g=128)
+    packed = layer.pack()
+    assert isinstance(packed, PackedTernaryLinear)
+    nbytes = sum(b.numel() * b.element_size() for b in packed.buffers())
+    assert nbytes == 520 * 1024 // 4 + 520 * (1024 // 128) * 4  # 0.25 + 4/g bytes per weight
+    x = torch.randn(2, m, 1024, device="cuda").to(torch.bfloat16)
+    with torch.no_grad():
+        y_train = layer(x)
+    y_packed = packed(x)
+    tq.device_status()
+    assert y_packed.shape == (2, m, 520) and y_packed.dtype == torch.bfloat16
+    assert torch.equal(y_packed, y_train)
