@@ -249,10 +249,9 @@ __device__ __forceinline__ uint32_t half_scale_x2(float s) {
   return u | (u << 16);
 }
 
-// Wait, with cluster-scope acquire, for a phase completed by arrivals from other
-// CTAs of the cluster (mbar_arrive_remote, a cluster-scope release), so that this
-// thread's later reads of their shared memory see what they wrote before
-// arriving. Gives up like mbar_wait.
+// Wait, with cluster-scope acquire, for a phase completed from other CTAs of the
+// cluster (the bytes of their st.async stores into this CTA's shared memory), so
+// that this thread's later reads see those bytes. Gives up like mbar_wait.
 __device__ __forceinline__ bool mbar_test_wait_cluster(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -372,7 +371,8 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
   auto rfull_bar = [&](int w, int p) { return bars + 160 + 8 * (2 * w + p); };
   auto rempty_bar = [&](int w, int p) { return bars + 288 + 8 * (2 * w + p); };
   // pieces of k: in the first CTA of a cluster, "the other CTAs' partial sums of
-  // row warp w are written"; in the others, "the first CTA has read them"
+  // row warp w have landed"; in the others, "the first CTA has them all" (this CTA
+  // may leave)
   auto xfull_bar = [&](int w) { return bars + 416 + 8 * w; };
   auto xdone_bar = [&](int w) { return bars + 896 + 8 * w; };
   SegInfo* info = reinterpret_cast<SegInfo*>(head + 512);  // kMaxStages x 48 bytes
