@@ -383,7 +383,10 @@ TQ_API tq_status tq_device_status(void* stream);
  *      release its first stage, so the producer's wait for that slot runs out;
  *   2  the dW product of tq_linear_bwd: the first epilogue warp of the first CTA
  *      pair's leader does not release its first accumulator, so the MMA issuer's
- *      wait for it runs out.
+ *      wait for it runs out;
+ *   4  a decode launch cut into pieces of k (tq_linear_fwd, m <= 16, fewer blocks
+ *      of 256 rows than SMs): CTA 1 sends none of its partial sums, so the first
+ *      CTA of its cluster waits for them in vain, and CTA 1 then for its release.
  * A launch made while a flag is set winds down at the limit (no copy or MMA left
  * in flight, every wait bounded) and reports TQ_ERR_TIMEOUT through
  * tq_device_status(); its outputs are undefined. Synchronises the device first.

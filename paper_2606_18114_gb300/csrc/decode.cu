@@ -343,6 +343,10 @@ __device__ __forceinline__ int find_mat(const DecodeBatch& b, int u) {
 constexpr int kSchedSlots = 256;
 __device__ uint32_t g_dsched[kSchedSlots][2];
 
+// Test flag (tq_test_hooks, DeviceCtl word 1): in a launch cut into pieces of k, CTA 1
+// sends none of its partial sums, so its cluster's first CTA waits for them in vain.
+constexpr int kWithholdDecodePieces = 4;
+
 // kPieces: a launch that cuts k into pieces (clusters; b.pieces > 1); without it
 // the persistent grid, compiled with none of the pieces' code.
 template <bool kTwoTiles, bool F16, bool kPieces>
@@ -902,8 +906,10 @@ __global__ void __launch_bounds__(DecodeCfg<kTwoTiles>::kThreads, 1)
         const uint32_t dst = map_to_rank(
             smem_u32(xpart + (((rank - 1) * kRowWarps + wr) * 32 + lane) * kLane), 0);
         const uint32_t bar = map_to_rank(xfull_bar(wr), 0);
+        // timeout tests only: CTA 1 withholds its partial sums
+        const bool withhold = blockIdx.x == 1 && test_withhold(status, kWithholdDecodePieces);
 #pragma unroll
-        for (int r = 0; r < kTiles; ++r) {
+        for (int r = 0; r < kTiles && !withhold; ++r) {
           if (v0) st_async_f4(dst + 16 * r, make_float4(acc[r][0], acc[r][1], acc[r][2], acc[r][3]), bar);
           if (v1)
             st_async_f4(dst + 16 * (2 + r), make_float4(acc1[r][0], acc1[r][1], acc1[r][2], acc1[r][3]),

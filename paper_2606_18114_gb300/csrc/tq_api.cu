@@ -771,7 +771,7 @@ TQ_API tq_status tq_device_status(void* stream) {
 TQ_API tq_status tq_test_hooks(int64_t wait_limit_ns, uint32_t flags) {
   g_err[0] = 0;
   if (wait_limit_ns < 0) return fail(TQ_ERR_INVALID_ARG, "negative wait limit");
-  if ((flags & ~3u) != 0) return fail(TQ_ERR_INVALID_ARG, "unknown test flags 0x%x", flags);
+  if ((flags & ~7u) != 0) return fail(TQ_ERR_INVALID_ARG, "unknown test flags 0x%x", flags);
   const DeviceInfo* dev = nullptr;
   TQ_TRY(device_info(&dev));
   cudaError_t e = cudaDeviceSynchronize();  // no kernel may be reading the words

@@ -238,5 +238,5 @@ def test_activation_flag_checked(lib):
 def test_test_hooks_reject_before_device(lib):
     # argument errors come before any device access
     assert lib.tq_test_hooks(-1, 0) == 1
-    assert lib.tq_test_hooks(1000, 4) == 1
+    assert lib.tq_test_hooks(1000, 8) == 1
     assert b"flags" in lib.tq_last_error()

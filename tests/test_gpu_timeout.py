@@ -96,6 +96,29 @@ def test_dw_withheld_accumulator_times_out_then_recovers(tq):
         assert torch.equal(got, ref)
 
 
+def test_decode_pieces_withheld_partial_sums_time_out_then_recover(tq):
+    """A decode cut into pieces of k (in_proj at one token: clusters of CTAs over each
+    block of rows): CTA 1 sends no partial sums, the first CTA of its cluster gives up
+    waiting for them, the others give up waiting for its release; every other cluster
+    finishes. The next normal calls give the clean result bit for bit."""
+    n, k, m, g = 8512, 2048, 1, 128
+    w = torch.from_numpy(synth.latent_weights(n, k, seed=85)).cuda()
+    x = synth.activations_bf16(m, k, seed=85).cuda()
+    codes, s, _ = tq.quantize(w, g)
+    ref = tq.linear_fwd(x, codes, s, g)
+    tq.device_status()
+    try:
+        tq.test_hooks(LIMIT_NS, 4)
+        tq.linear_fwd(x, codes, s, g)
+        _expect_timeout(tq)
+    finally:
+        tq.test_hooks(0, 0)
+    for _ in range(2):
+        got = tq.linear_fwd(x, codes, s, g)
+        tq.device_status()
+        assert torch.equal(got, ref)
+
+
 def test_hooks_off_by_default_after_reset(tq):
     """With the limit and flags reset, a normal launch reports no timeout."""
     tq.test_hooks(0, 0)
