@@ -109,3 +109,47 @@ def test_window_float2_loads_stay_paired_and_bank_conflict_free():
         banks = [kernel_window_index(gl, q0, gl) % 32 for gl in range(8)]
         words = {b for b in banks} | {b + 1 for b in banks}
         assert len(words) == 16
+
+
+def producer_windows(s0, s1, log2g):
+    """(segment, first group of the box) of every window load of a piece."""
+    wmask = (1 << (log2g - 4)) - 1
+    return [(s, (s >> (log2g - 4)) * WIN_GROUPS) for s in range(s0, s1)
+            if s == s0 or (s & wmask) == 0]
+
+
+def consumer_windows(s0, s1, log2g):
+    """(segment opening, segment closing) of every window the consumer waits for."""
+    wmask = (1 << (log2g - 4)) - 1
+    opened, out = None, []
+    for s in range(s0, s1):
+        if s == s0 or (s & wmask) == 0:
+            assert opened is None, "a window opened before the previous one closed"
+            opened = s
+        if (s & wmask) == wmask or s + 1 == s1:
+            out.append((opened, s))
+            opened = None
+    assert opened is None
+    return out
+
+
+@pytest.mark.parametrize("log2g", [5, 6, 7, 8, 9])
+def test_window_sequences_of_pieces_match(log2g):
+    g = 1 << log2g
+    for k in (g * 36, g * 64, g * 100 + 0):
+        k -= k % 64
+        nseg = (k + SEG_K - 1) // SEG_K
+        for pieces in (1, 2, 4, 8):
+            if pieces > nseg:
+                continue
+            for p in range(pieces):
+                s0, s1 = p * nseg // pieces, (p + 1) * nseg // pieces
+                loads = producer_windows(s0, s1, log2g)
+                waits = consumer_windows(s0, s1, log2g)
+                assert len(loads) == len(waits)           # one buffer use per window
+                for (ls, q0), (a, b) in zip(loads, waits):
+                    assert ls == a and q0 % 4 == 0         # TMA x: a multiple of 16 bytes
+                    for s in range(a, b + 1):              # every group the segment reads
+                        first = (s * SEG_K) >> log2g
+                        last = min(((s + 1) * SEG_K - 1) >> log2g, k // g - 1)
+                        assert q0 <= first and last < q0 + WIN_GROUPS
